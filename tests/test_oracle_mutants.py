@@ -1,0 +1,93 @@
+"""Plant plausible mistakes in copies of ``oracle/oracle.c`` and check that the
+pins catch every one.
+
+Each mutant is a textual substitution inside one function of the oracle's
+source.  The mutated copy is compiled with gcc into a temporary directory and
+run through all pins of its kind; at least one pin must fail.  If a
+substitution no longer matches the source (the oracle was edited), the test
+fails so that the mutant list is kept in step with the code.
+
+Every mutant keeps all memory accesses in bounds, so a broken copy can only
+give wrong numbers, never crash the test process.
+"""
+import re
+
+import pytest
+
+import oracle
+from _pins import ATTENTION_PINS, STAGE_PINS
+
+ATT = "oracle_decode_attention"
+STAGE = "oracle_prefix_stage"
+LOAD = "oracle_prefix_load"
+
+MUTANTS = [
+    # (id, function, old, new, count) -- count 0 replaces every occurrence
+    ("drop_softmax_scale", ATT,
+     "const double scale = 1.0 / sqrt((double)head_dim);", "const double scale = 1.0;", 1),
+    ("scale_by_d_not_sqrt_d", ATT,
+     "1.0 / sqrt((double)head_dim)", "1.0 / (double)head_dim", 1),
+    ("gqa_interleaved_heads", ATT,
+     "const int64_t g = h / group;", "const int64_t g = h % num_kv_heads;", 1),
+    ("query_indexed_by_kv_head", ATT,
+     "q + (b * num_q_heads + h) * head_dim", "q + (b * num_q_heads + g) * head_dim", 1),
+    ("slot_reversed_for_keys", ATT,
+     "const int64_t slot = t % page_size;",
+     "const int64_t slot = (page_size - 1) - t % page_size;", 1),
+    ("pages_in_reverse_order", ATT,
+     "block_table[b * max_pages + t / page_size]",
+     "block_table[b * max_pages + ((n + page_size - 1) / page_size - 1 - t / page_size)]", 0),
+    ("last_token_dropped", ATT,
+     "for (int64_t t = 0; t < n; ++t) {", "for (int64_t t = 0; t + 1 < n; ++t) {", 0),
+    ("exponent_sign_flipped", ATT, "exp(s[t] - m)", "exp(m - s[t])", 1),
+    ("values_read_from_keys", ATT, "v_pages + ((phys", "k_pages + ((phys", 1),
+    ("normalised_by_length", ATT, "o[d] /= l;", "o[d] /= (double)n;", 1),
+    ("lse_without_max", ATT, "lse[i] = m + log(l);", "lse[i] = log(l);", 1),
+    ("lse_base_two", ATT, "lse[i] = m + log(l);", "lse[i] = m + log2(l);", 1),
+    ("empty_lse_zero", ATT, "lse[i] = -INFINITY;", "lse[i] = 0.0;", 1),
+    ("stage_k_v_swapped", STAGE, "(kv == 0 ? k_pool : v_pool)", "(kv == 1 ? k_pool : v_pool)", 1),
+    ("stage_rows_head_major", STAGE,
+     "(((l - layer_begin) * 2 + kv) * num_kv_heads + h)",
+     "((h * (layer_end - layer_begin) + (l - layer_begin)) * 2 + kv)", 1),
+    ("stage_slot_reversed", STAGE,
+     "const int64_t slot = t % page_size;",
+     "const int64_t slot = (page_size - 1) - t % page_size;", 1),
+    ("stage_wrong_layer", STAGE, "+ l * layer_stride", "+ (l - layer_begin) * layer_stride", 1),
+    ("stage_packed_offset_one_layer", STAGE,
+     "layers * 2 * num_kv_heads * head_dim", "2 * num_kv_heads * head_dim", 1),
+    ("load_tokens_reversed", LOAD,
+     "memcpy(d, row + t * head_dim", "memcpy(d, row + (n - 1 - t) * head_dim", 1),
+    ("load_k_v_swapped", LOAD, "(kv == 0 ? k_pool : v_pool)", "(kv == 1 ? k_pool : v_pool)", 1),
+]
+
+
+def _function_span(src: str, name: str):
+    m = re.search(r"^int " + name + r"\(", src, flags=re.M)
+    assert m, f"function {name} not found in oracle.c"
+    end = src.index("\n}\n", m.start())
+    return m.start(), end
+
+
+def mutate(src: str, func: str, old: str, new: str, count: int) -> str:
+    a, b = _function_span(src, func)
+    body = src[a:b]
+    assert old in body, f"mutation anchor {old!r} not found in {func}"
+    body = body.replace(old, new) if count == 0 else body.replace(old, new, count)
+    return src[:a] + body + src[b:]
+
+
+@pytest.mark.parametrize("mid,func,old,new,count", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_pins_catch_mutant(tmp_path, mid, func, old, new, count):
+    src = oracle.SOURCE.read_text()
+    path = tmp_path / f"{mid}.c"
+    path.write_text(mutate(src, func, old, new, count))
+    lib = oracle.compile_library(path, tmp_path / f"lib{mid}.so")
+    orc = oracle.Oracle(lib)
+    pins = ATTENTION_PINS if func == ATT else STAGE_PINS
+    caught = []
+    for pin in pins:
+        try:
+            pin(orc)
+        except (AssertionError, oracle.OracleError, ValueError, FloatingPointError):
+            caught.append(pin.__name__)
+    assert caught, f"mutant {mid} survived every pin"
