@@ -1,0 +1,546 @@
+"""Benchmark: batched paged-KV decode attention on one GB300 (per rank).
+
+Headline workload: the mixed heavy-tailed rollout batch -- 512 trajectories,
+context lengths lognormal (median 4096, sigma 1) clipped to [512, 131072],
+64 query / 8 KV heads, head dim 128, 16-token pages in a shuffled pool (about
+14 GB of bf16 KV, far larger than L2).  A step is one decode_attention call
+over the whole batch for one layer: the planner launch plus the attention
+launch (the split-KV merge runs inside the attention kernel).
+
+Printed: one JSON line with the achieved HBM GB/s of algorithmic bytes
+(K and V of every context token once per KV head, plus q, out, lse, the
+block-table entries used and context_lens), decode steps/s, the attention
+kernel's roofline fraction, an end-to-end number through the C ABI with
+host buffers, the fp64 CPU oracle timed on a bounded sample, SM clocks
+during the timed region and, as a secondary measurement, prefix staging.
+
+``--impl reference`` times the oracle (the CPU reference of this build) on
+the same workload and prints the same metric.
+Multi-GPU (torchrun): each rank runs its own batch (weak scaling, no
+collective on the data path); rank 0 prints the whole-job numbers.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import paper_2609_36899_gb300 as cadkv  # noqa: E402
+from paper_2609_36899_gb300 import build as pkg_build  # noqa: E402
+from paper_2609_36899_gb300.workloads import (DECODE_WORKLOADS, STAGING, bf16_bits,  # noqa: E402
+                                              fill_layer_pool, make_decode_batch,
+                                              make_staging_job)
+
+METRIC = "decode-attention achieved HBM GB/s (% of 8 TB/s) and decode steps/s per batch"
+NOMINAL_HBM_GBS = 8000.0
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_HBM_GBS = 6800.0
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "decode_attention_mixed_b512.md")
+STAGE_PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "prefix_stage_copy_64traj.md")
+KERNEL_SOURCE = os.path.join(ROOT, "paper_2609_36899_gb300", "csrc", "decode_attention.cu")
+STAGE_SOURCE = os.path.join(ROOT, "paper_2609_36899_gb300", "csrc", "prefix_stage.cu")
+
+
+# ------------------------------------------------------------------ helpers
+
+def hbm_peak():
+    try:
+        with open(PEAKS_FILE) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def source_hash(path):
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def profiled_traffic(summary_path, source_path):
+    """DRAM bytes per launch from a committed ncu summary, or None when the
+    summary is missing or was taken on a different kernel source."""
+    try:
+        text = open(summary_path).read()
+    except OSError:
+        return None
+    m = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]{16})", text)
+    t = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    if not m or not t or m.group(1) != source_hash(source_path):
+        return None
+    return float(t.group(1))
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons every 200 ms."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device):
+        self.proc = None
+        try:
+            self.gpu_id = "GPU-" + str(torch.cuda.get_device_properties(device).uuid)
+        except Exception:
+            self.gpu_id = str(device.index or 0)
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu_id}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, sm_max, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                sm_max.append(float(parts[1]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[4:8]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(sm_max),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def decode_bytes(lens, hq, hkv, d):
+    """Algorithmic bytes of one decode step (see module docstring)."""
+    lens = np.asarray(lens, dtype=np.int64)
+    b = len(lens)
+    pages = int((-(-lens // 16)).sum())
+    kv = 4 * hkv * d * int(lens.sum())
+    qo = 2 * (2 * b * hq * d)
+    return kv + qo + 4 * b * hq + 4 * pages + 4 * b
+
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(0)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64,
+                     device="cuda" if dist.get_backend() == "nccl" else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64,
+                     device="cuda" if dist.get_backend() == "nccl" else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------ CPU oracle leg
+
+class OracleSample:
+    """A bounded sample of a batch's trajectories, copied to the host once, on
+    which the fp64 oracle is timed.
+
+    Trajectories are taken in a seeded shuffled order until the estimated
+    oracle time (from a one-trajectory pilot) reaches ``target_s``.
+    """
+
+    def __init__(self, batch, target_s: float, threads: int | None = None):
+        import oracle
+        oracle.build()
+        self.orc = oracle.default()
+        self.threads = threads or len(os.sched_getaffinity(0))
+        w = batch.workload
+        lens = batch.context_lens
+        order = np.random.Generator(np.random.PCG64(w.seed + 99)).permutation(len(lens))
+        pilot = self._inputs(batch, [int(order[0])])
+        t = self._time(pilot)
+        budget_tokens = max(int(lens[order[0]]), 1) / max(t, 1e-6) * target_s
+        chosen, tokens = [], 0
+        for b in order:
+            chosen.append(int(b))
+            tokens += int(lens[b])
+            if tokens >= budget_tokens:
+                break
+        self.inputs = self._inputs(batch, chosen)
+        sel = lens[np.array(chosen)]
+        self.nbytes = decode_bytes(sel, w.num_q_heads, w.num_kv_heads, w.head_dim)
+        self.desc = (f"{len(chosen)} of {len(lens)} trajectories of the same batch "
+                     f"({int(sel.sum())} context tokens, all {w.num_q_heads} query heads), "
+                     f"fp64 oracle, OpenMP {self.threads} threads")
+
+    @staticmethod
+    def _inputs(batch, chosen):
+        lens = batch.context_lens[np.array(chosen)]
+        pages = -(-lens.astype(np.int64) // 16)
+        phys = np.concatenate([batch.block_table[b, :p] for b, p in zip(chosen, pages)])
+        idx = torch.from_numpy(phys.astype(np.int64)).to(batch.k_pages.device)
+        k = bf16_bits(batch.k_pages.index_select(0, idx))
+        v = bf16_bits(batch.v_pages.index_select(0, idx))
+        q = bf16_bits(batch.q[torch.as_tensor(chosen, device=batch.q.device)])
+        table = np.full((len(chosen), max(int(pages.max()), 1)), -1, dtype=np.int32)
+        pos = 0
+        for i, p in enumerate(pages):
+            table[i, :p] = np.arange(pos, pos + p)
+            pos += p
+        return q, k, v, table, lens
+
+    def _time(self, inputs):
+        t0 = time.perf_counter()
+        self.orc.decode_attention(*inputs, num_threads=self.threads)
+        return time.perf_counter() - t0
+
+    def run(self) -> float:
+        """Seconds for one oracle evaluation of the sample."""
+        return self._time(self.inputs)
+
+
+# ------------------------------------------------------------------ GPU legs
+
+def time_decode(tensors, steps, warmup, stream):
+    q, k, v, bt, cl, out, lse, ws = tensors
+    for _ in range(warmup):
+        cadkv.decode_attention_plan(q, k, v, bt, cl, out, lse, ws, stream=stream)
+        cadkv.decode_attention_run(q, k, v, bt, cl, out, lse, ws, stream=stream)
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    return ev
+
+
+def run_decode_loop(tensors, ev, stream):
+    q, k, v, bt, cl, out, lse, ws = tensors
+    for e0, e1, e2 in ev:
+        e0.record(stream)
+        cadkv.decode_attention_plan(q, k, v, bt, cl, out, lse, ws, stream=stream)
+        e1.record(stream)
+        cadkv.decode_attention_run(q, k, v, bt, cl, out, lse, ws, stream=stream)
+        e2.record(stream)
+
+
+def e2e_loop(batch, tensors, steps, warmup, stream):
+    """decode_attention through the C ABI with host inputs and outputs: every
+    step copies q, block_table and context_lens from pinned host memory, runs
+    the step and reads out and lse back to pinned host memory."""
+    q, k, v, bt, cl, out, lse, ws = tensors
+    hq = batch.q.cpu().pin_memory()
+    hbt = torch.from_numpy(batch.block_table).pin_memory()
+    hcl = torch.from_numpy(batch.context_lens).pin_memory()
+    hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    hlse = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
+
+    def step():
+        with torch.cuda.stream(stream):
+            q.copy_(hq, non_blocking=True)
+            bt.copy_(hbt, non_blocking=True)
+            cl.copy_(hcl, non_blocking=True)
+            cadkv.decode_attention(q, k, v, bt, cl, out=out, lse=lse, workspace=ws,
+                                   stream=stream)
+            hout.copy_(out, non_blocking=True)
+            hlse.copy_(lse, non_blocking=True)
+        stream.synchronize()
+
+    for _ in range(warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        step()
+    secs = (time.perf_counter() - t0) / steps
+    h2d = hq.numel() * 2 + hbt.numel() * 4 + hcl.numel() * 4
+    d2h = hout.numel() * 2 + hlse.numel() * 4
+    return secs, h2d, d2h
+
+
+def bench_staging(device, reps, layers=2):
+    """Prefix staging of all 64 trajectories of the staging workload for
+    ``layers`` layers (the full 48-layer job does not fit in HBM next to its
+    destination; it runs as 48 / layers such chunks)."""
+    job = make_staging_job(STAGING)
+    k_layers = [torch.empty((job.num_pages, 8, 16, 128), dtype=torch.bfloat16, device=device)
+                for _ in range(layers)]
+    v_layers = [torch.empty_like(k_layers[0]) for _ in range(layers)]
+    for l in range(layers):
+        fill_layer_pool(k_layers[l], v_layers[l], STAGING.seed, l)
+    pool = cadkv.KVPool(k_layers, v_layers)
+    lens = job.context_lens
+    size = cadkv.staged_size(lens, 0, layers, 8, 128)
+    dst = torch.empty(size, dtype=torch.bfloat16, device=device)
+    bt = torch.from_numpy(job.block_table).to(device)
+    cl = torch.from_numpy(lens).to(device)
+    ws = torch.empty(cadkv.kv_prefix_stage_workspace_size(len(lens)), dtype=torch.uint8,
+                     device=device)
+    stream = torch.cuda.current_stream(device)
+    for _ in range(3):
+        cadkv.kv_prefix_stage(pool, bt, cl, 0, layers, dst, workspace=ws, stream=stream)
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(reps)]
+    for e0, e1 in ev:
+        e0.record(stream)
+        cadkv.kv_prefix_stage(pool, bt, cl, 0, layers, dst, workspace=ws, stream=stream)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    status = cadkv.kv_prefix_stage_status(ws)
+    ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in ev)
+    moved = 2 * size * 2  # read + write, bytes
+    # bit-exact spot check of one trajectory's staged rows against the pool
+    b = int(np.argmax(lens))
+    p = -(-int(lens[b]) // 16)
+    starts = np.concatenate([[0], np.cumsum(lens.astype(np.int64) * layers * 2 * 8 * 128)])
+    got = dst[int(starts[b]):int(starts[b + 1])].view(layers, 2, 8, int(lens[b]), 128)
+    phys = bt[b, :p].long()
+    ok = True
+    for l in range(layers):
+        for kv, src in ((0, k_layers[l]), (1, v_layers[l])):
+            rows = src.index_select(0, phys).permute(1, 0, 2, 3).reshape(8, p * 16, 128)
+            ok &= bool(torch.equal(rows[:, :int(lens[b])].view(torch.int16),
+                                   got[l, kv].view(torch.int16)))
+    peak, kind = hbm_peak()
+    gbs = moved / (ms * 1e-3) / 1e9
+    res = {"workload": f"{STAGING.name}: 64 trajectories, {layers} of 48 layers per call",
+           "gbps_read_plus_write": round(gbs, 1), "ms_per_call": round(ms, 3),
+           "bytes_per_call": moved, "launches_per_call": 2, "status": status,
+           "bit_exact_spot_check": ok,
+           "full_job_ms_estimate": round(ms * 48 / layers, 1),
+           "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": peak,
+                        "unit": "GB/s", "frac": round(gbs / peak, 4),
+                        "peak_kind": kind,
+                        "traffic": profiled_traffic(STAGE_PROFILE_SUMMARY, STAGE_SOURCE)}}
+    del dst, k_layers, v_layers, pool
+    torch.cuda.empty_cache()
+    return res
+
+
+def bench_config(name, device, steps, warmup):
+    w = DECODE_WORKLOADS[name]
+    batch = make_decode_batch(w, device=device)
+    tensors = _tensors(batch, device)
+    stream = torch.cuda.current_stream(device)
+    ev = time_decode(tensors, steps, warmup, stream)
+    run_decode_loop(tensors, ev, stream)
+    torch.cuda.synchronize()
+    step_ms = ev[0][0].elapsed_time(ev[-1][2]) / steps
+    kern_ms = statistics.mean(e1.elapsed_time(e2) for _, e1, e2 in ev)
+    nbytes = decode_bytes(batch.context_lens, w.num_q_heads, w.num_kv_heads, w.head_dim)
+    res = {"gbps": round(nbytes / (step_ms * 1e-3) / 1e9, 1),
+           "steps_per_s": round(1e3 / step_ms, 1), "ms_per_step": round(step_ms, 4),
+           "attention_kernel_gbps": round(nbytes / (kern_ms * 1e-3) / 1e9, 1)}
+    del batch, tensors
+    torch.cuda.empty_cache()
+    return res
+
+
+def _tensors(batch, device):
+    w = batch.workload
+    q = batch.q.to(device)
+    k = batch.k_pages.to(device)
+    v = batch.v_pages.to(device)
+    bt = torch.from_numpy(batch.block_table).to(device)
+    cl = torch.from_numpy(batch.context_lens).to(device)
+    out = torch.empty_like(q)
+    lse = torch.empty((len(batch.context_lens), w.num_q_heads), dtype=torch.float32,
+                      device=device)
+    ws = torch.empty(cadkv.decode_attention_workspace_size(len(batch.context_lens), w.num_q_heads,
+                                                           w.num_kv_heads, w.head_dim,
+                                                           bt.shape[1]),
+                     dtype=torch.uint8, device=device)
+    return q, k, v, bt, cl, out, lse, ws
+
+
+# ------------------------------------------------------------------ main
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=sorted(DECODE_WORKLOADS), default="mixed")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target oracle time of the cpu_baseline sample")
+    ap.add_argument("--reference-seconds", type=float, default=90.0,
+                    help="target total oracle time of the --impl reference run")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the staging and other-workload secondary measurements")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+
+    world, rank, local = dist_setup(args)
+    if args.impl == "reference":
+        return reference_arm(args, world, rank)
+
+    pkg_build.build()
+    device = torch.device("cuda", torch.cuda.current_device())
+    w = DECODE_WORKLOADS[args.workload]
+    batch = make_decode_batch(w, device=device, seed=w.seed + rank)
+    tensors = _tensors(batch, device)
+    stream = torch.cuda.current_stream(device)
+    nbytes = decode_bytes(batch.context_lens, w.num_q_heads, w.num_kv_heads, w.head_dim)
+
+    ev = time_decode(tensors, args.steps, args.warmup, stream)
+    sampler = ClockSampler(device)
+    barrier(world)
+    torch.cuda.synchronize()
+    sampler.start()
+    run_decode_loop(tensors, ev, stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clocks = sampler.stop()
+    status = cadkv.decode_attention_status(tensors[7])
+
+    total_ms = ev[0][0].elapsed_time(ev[-1][2])
+    kern_ms = statistics.mean(e1.elapsed_time(e2) for _, e1, e2 in ev)
+    plan_ms = statistics.mean(e0.elapsed_time(e1) for e0, e1, _ in ev)
+    total_ms = max_over_ranks(total_ms, world)
+    step_ms = total_ms / args.steps
+    all_bytes = sum_over_ranks(float(nbytes), world)
+    value = all_bytes * args.steps / (total_ms * 1e-3) / 1e9
+
+    e2e_s, h2d, d2h = e2e_loop(batch, tensors, max(args.steps // 4, 20), 3, stream)
+    e2e_s = max_over_ranks(e2e_s, world)
+    e2e_value = all_bytes / e2e_s / 1e9
+
+    peak, kind = hbm_peak()
+    achieved = nbytes / (kern_ms * 1e-3) / 1e9
+    line = {
+        "metric": METRIC,
+        "value": round(value, 1),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(step_ms, 4),
+        "steps_per_s": round(1e3 / step_ms, 2),
+        "pct_of_8tbps": round(100 * value / world / NOMINAL_HBM_GBS, 2),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": w.name, "batch": len(batch.context_lens),
+                   "context_lens": "lognormal median 4096 sigma 1.0 clipped [512, 131072]"
+                   if args.workload == "mixed" else str(w.length_args),
+                   "total_context_tokens": int(batch.context_lens.sum()),
+                   "num_q_heads": w.num_q_heads, "num_kv_heads": w.num_kv_heads,
+                   "head_dim": w.head_dim, "page_size": 16,
+                   "kv_pool_gb": round(2 * batch.k_pages.numel() * 2 / 1e9, 2),
+                   "bytes_per_step": nbytes, "layers_per_step": 1,
+                   "l2": "inputs larger than L2 (no flush)",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "e2e": {"value": round(e2e_value, 1), "unit": "GB/s",
+                "ms_per_step": round(e2e_s * 1e3, 4),
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": 2 * args.steps,
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+                     "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "peak_kind": kind, "kernel": "decode_attention_kernel<128>",
+                     "kernel_ms": round(kern_ms, 4), "planner_ms": round(plan_ms, 4),
+                     "traffic": profiled_traffic(PROFILE_SUMMARY, KERNEL_SOURCE)},
+        "clocks": clocks,
+        "device_status": status,
+    }
+    if rank == 0 and not args.no_extras:
+        extras = {}
+        for other in ("paced", "long_tail"):
+            if other != args.workload:
+                extras[other] = bench_config(other, device, max(args.steps // 4, 50), 5)
+        line["other_workloads"] = extras
+    if rank == 0 and not args.no_cpu_baseline:
+        sample = OracleSample(batch, args.cpu_seconds)
+        secs = sample.run()
+        line["cpu_baseline"] = {"value": round(sample.nbytes / secs / 1e9, 4), "unit": "GB/s",
+                                "cores": sample.threads, "kind": "oracle",
+                                "sample": sample.desc, "seconds": round(secs, 2)}
+    del batch, tensors
+    torch.cuda.empty_cache()
+    if rank == 0 and not args.no_extras:
+        line["staging"] = bench_staging(device, reps=10)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def reference_arm(args, world, rank):
+    """The oracle, as it stands, on the host cores: same metric and workload,
+    each step one oracle evaluation of a bounded sample of the same batch,
+    sized so that warm-up plus timed steps take about --reference-seconds."""
+    if rank != 0:
+        return
+    w = DECODE_WORKLOADS[args.workload]
+    device = torch.device("cuda", 0) if torch.cuda.is_available() else torch.device("cpu")
+    batch = make_decode_batch(w, device=device)
+    per_step = min(max(args.reference_seconds / (args.steps + args.warmup), 0.02), 10.0)
+    sample = OracleSample(batch, per_step)
+    for _ in range(args.warmup):
+        sample.run()
+    secs = sum(sample.run() for _ in range(args.steps))
+    value = sample.nbytes * args.steps / secs / 1e9
+    line = {"metric": METRIC, "value": round(value, 4), "unit": "GB/s", "impl": "reference",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1e3 * secs / args.steps, 2),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": w.name, "batch": len(batch.context_lens),
+                       "num_q_heads": w.num_q_heads, "num_kv_heads": w.num_kv_heads,
+                       "head_dim": w.head_dim, "page_size": 16},
+            "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": sample.threads,
+                             "kind": "oracle", "sample": "per step: " + sample.desc},
+            "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,526 @@
+// capi.cu -- the extern "C" entry points declared in include/cadkv.h.
+//
+// Host side only: argument validation, workspace carving, TMA tensor-map
+// encoding and kernel launches.  Every numeric step runs in the kernels of
+// decode_attention.cu and prefix_stage.cu.
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <vector>
+
+#include "internal.h"
+
+using namespace cadkv;
+
+struct cadkv_pool {
+    int num_layers = 0, num_pages = 0, page_size = 0, num_kv_heads = 0, head_dim = 0;
+    int device = 0;
+    void *owned = nullptr;          // single allocation holding all pages, if owned
+    void **dev_layer_ptrs = nullptr;  // device array [2 * num_layers]: K pointers then V
+    std::vector<void *> k, v;
+};
+
+namespace {
+
+constexpr int kAbiVersion = (1 << 16) | 0;
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+int device_sms()
+{
+    static std::mutex mu;
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0)
+        return CADKV_ERR_CUDA;
+    if (dev < 64) {
+        std::lock_guard<std::mutex> lock(mu);
+        if (cache[dev] > 0)
+            return cache[dev];
+    }
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
+        return CADKV_ERR_CUDA;
+    if (dev < 64) {
+        std::lock_guard<std::mutex> lock(mu);
+        cache[dev] = sms;
+    }
+    return sms;
+}
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                   const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                   const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled_fn()
+{
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    });
+    return fn;
+}
+
+// Tensor map over one layer's pages viewed as a 2-D bf16 matrix
+// [num_pages * Hkv * 16 rows][D columns]; box = 16 rows x 64 columns (128 B),
+// 128-byte swizzle so that ldmatrix reads of a page are bank-conflict free.
+int encode_pages_map(CUtensorMap *map, const void *pages, int num_pages, int num_kv_heads,
+                     int head_dim)
+{
+    EncodeTiledFn fn = encode_tiled_fn();
+    if (!fn)
+        return CADKV_ERR_CUDA;
+    const cuuint64_t dims[2] = {(cuuint64_t)head_dim,
+                                (cuuint64_t)num_pages * num_kv_heads * kPageSize};
+    const cuuint64_t strides[1] = {(cuuint64_t)head_dim * 2};
+    const cuuint32_t box[2] = {64, (cuuint32_t)kPageSize};
+    const cuuint32_t elem[2] = {1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(pages), dims,
+                    strides, box, elem, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? CADKV_OK : CADKV_ERR_CUDA;
+}
+
+struct DecodeShape {
+    int batch, num_q_heads, num_kv_heads, head_dim, page_size, num_pages, max_pages;
+};
+
+int check_decode_shape(const DecodeShape &s)
+{
+    if (s.batch < 0 || s.num_q_heads <= 0 || s.num_kv_heads <= 0 || s.max_pages < 0 ||
+        s.head_dim <= 0 || s.page_size <= 0)
+        return CADKV_ERR_SHAPE;
+    if (s.num_q_heads % s.num_kv_heads != 0)
+        return CADKV_ERR_SHAPE;
+    if (s.num_q_heads / s.num_kv_heads > kMaxGroup)
+        return CADKV_ERR_UNSUPPORTED;
+    if (s.head_dim != 64 && s.head_dim != 128)
+        return CADKV_ERR_UNSUPPORTED;
+    if (s.page_size != kPageSize)
+        return CADKV_ERR_UNSUPPORTED;
+    if ((long long)s.max_pages * kPageSize > INT32_MAX)
+        return CADKV_ERR_SHAPE;
+    return CADKV_OK;
+}
+
+int workspace_carve(const DecodeShape &s, void *workspace, size_t workspace_bytes, int sms,
+                    DecodeWorkspaceLayout *L)
+{
+    *L = decode_workspace_layout(s.batch, s.num_kv_heads, s.num_q_heads / s.num_kv_heads,
+                                 s.head_dim, sms);
+    if (!workspace || !aligned(workspace, kWorkspaceAlign) || workspace_bytes < L->total)
+        return CADKV_ERR_WORKSPACE;
+    return CADKV_OK;
+}
+
+int plan_impl(const int32_t *context_lens, void *out, float *lse, const DecodeShape &s,
+              int slice_pages, void *workspace, size_t workspace_bytes, cudaStream_t stream)
+{
+    int rc = check_decode_shape(s);
+    if (rc != CADKV_OK)
+        return rc;
+    if (s.batch == 0)
+        return CADKV_OK;
+    if (!context_lens || !out)
+        return CADKV_ERR_INVALID;
+    if (!aligned(out, 16) || !aligned(context_lens, 4) || (lse && !aligned(lse, 4)))
+        return CADKV_ERR_INVALID;
+    if (slice_pages < 0)
+        return CADKV_ERR_INVALID;
+    const int sms = device_sms();
+    if (sms < 0)
+        return sms;
+    DecodeWorkspaceLayout L;
+    rc = workspace_carve(s, workspace, workspace_bytes, sms, &L);
+    if (rc != CADKV_OK)
+        return rc;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    PlanParams p{};
+    p.context_lens = context_lens;
+    p.out = static_cast<__nv_bfloat16 *>(out);
+    p.lse = lse;
+    p.hdr = reinterpret_cast<WorkspaceHeader *>(ws);
+    p.page_prefix = reinterpret_cast<long long *>(ws + L.page_prefix);
+    p.unit_counter = reinterpret_cast<int *>(ws + L.unit_counter);
+    p.batch = s.batch;
+    p.num_q_heads = s.num_q_heads;
+    p.num_kv_heads = s.num_kv_heads;
+    p.head_dim = s.head_dim;
+    p.max_pages = s.max_pages;
+    p.slice_cap = L.slice_cap;
+    p.slice_pages = slice_pages;
+    return launch_plan(p, stream) == cudaSuccess ? CADKV_OK : CADKV_ERR_CUDA;
+}
+
+int check_run_args(const void *q, const void *k_pages, const void *v_pages,
+                   const int32_t *block_table, const int32_t *context_lens, const void *out,
+                   const float *lse, const DecodeShape &s)
+{
+    if (!q || !k_pages || !v_pages || !block_table || !context_lens || !out)
+        return CADKV_ERR_INVALID;
+    if (!aligned(q, 16) || !aligned(k_pages, 16) || !aligned(v_pages, 16) || !aligned(out, 16) ||
+        !aligned(block_table, 4) || !aligned(context_lens, 4) || (lse && !aligned(lse, 4)))
+        return CADKV_ERR_INVALID;
+    if (s.num_pages <= 0)
+        return CADKV_ERR_SHAPE;
+    if ((long long)s.num_pages * s.num_kv_heads * kPageSize > INT32_MAX)
+        return CADKV_ERR_UNSUPPORTED;
+    return CADKV_OK;
+}
+
+int run_impl(const void *q, const void *k_pages, const void *v_pages,
+             const int32_t *block_table, const int32_t *context_lens, void *out, float *lse,
+             const DecodeShape &s, void *workspace, size_t workspace_bytes, cudaStream_t stream)
+{
+    int rc = check_decode_shape(s);
+    if (rc != CADKV_OK)
+        return rc;
+    if (s.batch == 0)
+        return CADKV_OK;
+    rc = check_run_args(q, k_pages, v_pages, block_table, context_lens, out, lse, s);
+    if (rc != CADKV_OK)
+        return rc;
+    const int sms = device_sms();
+    if (sms < 0)
+        return sms;
+    DecodeWorkspaceLayout L;
+    rc = workspace_carve(s, workspace, workspace_bytes, sms, &L);
+    if (rc != CADKV_OK)
+        return rc;
+    CUtensorMap kmap, vmap;
+    if (encode_pages_map(&kmap, k_pages, s.num_pages, s.num_kv_heads, s.head_dim) != CADKV_OK ||
+        encode_pages_map(&vmap, v_pages, s.num_pages, s.num_kv_heads, s.head_dim) != CADKV_OK)
+        return CADKV_ERR_CUDA;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    AttnParams p{};
+    p.q = static_cast<const __nv_bfloat16 *>(q);
+    p.block_table = block_table;
+    p.context_lens = context_lens;
+    p.out = static_cast<__nv_bfloat16 *>(out);
+    p.lse = lse;
+    p.hdr = reinterpret_cast<WorkspaceHeader *>(ws);
+    p.page_prefix = reinterpret_cast<const long long *>(ws + L.page_prefix);
+    p.unit_counter = reinterpret_cast<int *>(ws + L.unit_counter);
+    p.part_lse = reinterpret_cast<float *>(ws + L.part_lse);
+    p.part_o = reinterpret_cast<float *>(ws + L.part_o);
+    p.batch = s.batch;
+    p.num_q_heads = s.num_q_heads;
+    p.num_kv_heads = s.num_kv_heads;
+    p.group = s.num_q_heads / s.num_kv_heads;
+    p.max_pages = s.max_pages;
+    p.num_pages = s.num_pages;
+    p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s.head_dim));
+    return launch_attention(p, kmap, vmap, s.head_dim, sms, stream) == cudaSuccess ? CADKV_OK
+                                                                                    : CADKV_ERR_CUDA;
+}
+
+int read_status(const void *workspace, cudaStream_t stream)
+{
+    if (!workspace)
+        return CADKV_ERR_INVALID;
+    int status = 0;
+    if (cudaMemcpyAsync(&status, workspace, sizeof(int), cudaMemcpyDeviceToHost, stream) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(stream) != cudaSuccess)
+        return CADKV_ERR_CUDA;
+    return status;
+}
+
+int stage_impl(const cadkv_pool *pool, const int32_t *block_table, int max_pages,
+               const int32_t *context_lens, int batch, int layer_begin, int layer_end,
+               const void *rows, const int64_t *offsets, void *workspace,
+               size_t workspace_bytes, cudaStream_t stream, int to_pool)
+{
+    if (!pool)
+        return CADKV_ERR_INVALID;
+    if (batch < 0 || max_pages < 0 || layer_begin < 0 || layer_end > pool->num_layers ||
+        layer_begin > layer_end)
+        return CADKV_ERR_SHAPE;
+    if ((long long)max_pages * kPageSize > INT32_MAX)
+        return CADKV_ERR_SHAPE;
+    if (batch == 0 || layer_begin == layer_end)
+        return CADKV_OK;
+    if (!block_table || !context_lens || !rows)
+        return CADKV_ERR_INVALID;
+    if (!aligned(rows, 16) || !aligned(block_table, 4) || !aligned(context_lens, 4) ||
+        (offsets && !aligned(offsets, 8)))
+        return CADKV_ERR_INVALID;
+    const StageWorkspaceLayout L = stage_workspace_layout(batch);
+    if (!workspace || !aligned(workspace, kWorkspaceAlign) || workspace_bytes < L.total)
+        return CADKV_ERR_WORKSPACE;
+    const int sms = device_sms();
+    if (sms < 0)
+        return sms;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    StageParams p{};
+    p.layer_k = pool->dev_layer_ptrs;
+    p.layer_v = pool->dev_layer_ptrs + pool->num_layers;
+    p.block_table = block_table;
+    p.context_lens = context_lens;
+    p.rows = const_cast<void *>(rows);
+    p.row_offsets = reinterpret_cast<const long long *>(offsets);
+    p.hdr = reinterpret_cast<WorkspaceHeader *>(ws);
+    p.page_prefix = reinterpret_cast<long long *>(ws + L.page_prefix);
+    p.token_prefix = reinterpret_cast<long long *>(ws + L.token_prefix);
+    p.unit_prefix = reinterpret_cast<long long *>(ws + L.unit_prefix);
+    p.batch = batch;
+    p.max_pages = max_pages;
+    p.num_pages = pool->num_pages;
+    p.num_kv_heads = pool->num_kv_heads;
+    p.head_dim = pool->head_dim;
+    p.layer_begin = layer_begin;
+    p.layer_end = layer_end;
+    p.to_pool = to_pool;
+    return launch_stage(p, sms, stream) == cudaSuccess ? CADKV_OK : CADKV_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *kv_status_string(int status)
+{
+    switch (status) {
+    case CADKV_OK: return "ok";
+    case CADKV_ERR_INVALID: return "invalid argument (null or misaligned pointer, bad value)";
+    case CADKV_ERR_SHAPE: return "inconsistent sizes or context length out of range";
+    case CADKV_ERR_CUDA: return "CUDA call failed";
+    case CADKV_ERR_UNSUPPORTED: return "unsupported head_dim, page_size or head group";
+    case CADKV_ERR_OOB: return "block-table entry outside the KV pool";
+    case CADKV_ERR_TIMEOUT: return "device-side wait timed out";
+    case CADKV_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    default: return "unknown status";
+    }
+}
+
+int cadkv_abi_version(void) { return kAbiVersion; }
+
+int cadkv_device_sms(void) { return device_sms(); }
+
+int kv_pool_create(cadkv_pool **out, int num_layers, int num_pages, int page_size,
+                   int num_kv_heads, int head_dim, void *const *k_layers, void *const *v_layers)
+{
+    if (!out)
+        return CADKV_ERR_INVALID;
+    *out = nullptr;
+    if (num_layers <= 0 || num_pages <= 0 || num_kv_heads <= 0)
+        return CADKV_ERR_SHAPE;
+    if (page_size != kPageSize || (head_dim != 64 && head_dim != 128))
+        return CADKV_ERR_UNSUPPORTED;
+    if ((k_layers == nullptr) != (v_layers == nullptr))
+        return CADKV_ERR_INVALID;
+    if (k_layers)
+        for (int l = 0; l < num_layers; ++l)
+            if (!k_layers[l] || !v_layers[l] || !aligned(k_layers[l], 16) ||
+                !aligned(v_layers[l], 16))
+                return CADKV_ERR_INVALID;
+    cadkv_pool *pool = new (std::nothrow) cadkv_pool;
+    if (!pool)
+        return CADKV_ERR_INVALID;
+    try {
+        pool->k.resize(num_layers);
+        pool->v.resize(num_layers);
+    } catch (...) {
+        delete pool;
+        return CADKV_ERR_INVALID;
+    }
+    pool->num_layers = num_layers;
+    pool->num_pages = num_pages;
+    pool->page_size = page_size;
+    pool->num_kv_heads = num_kv_heads;
+    pool->head_dim = head_dim;
+    cudaGetDevice(&pool->device);
+    const size_t layer_bytes = (size_t)num_pages * num_kv_heads * page_size * head_dim * 2;
+    if (k_layers) {
+        for (int l = 0; l < num_layers; ++l) {
+            pool->k[l] = k_layers[l];
+            pool->v[l] = v_layers[l];
+        }
+    } else {
+        if (cudaMalloc(&pool->owned, layer_bytes * 2 * num_layers) != cudaSuccess) {
+            delete pool;
+            return CADKV_ERR_CUDA;
+        }
+        for (int l = 0; l < num_layers; ++l) {
+            pool->k[l] = static_cast<uint8_t *>(pool->owned) + (size_t)(2 * l) * layer_bytes;
+            pool->v[l] = static_cast<uint8_t *>(pool->owned) + (size_t)(2 * l + 1) * layer_bytes;
+        }
+    }
+    std::vector<void *> ptrs(2 * (size_t)num_layers);
+    for (int l = 0; l < num_layers; ++l) {
+        ptrs[l] = pool->k[l];
+        ptrs[num_layers + l] = pool->v[l];
+    }
+    if (cudaMalloc(&pool->dev_layer_ptrs, ptrs.size() * sizeof(void *)) != cudaSuccess ||
+        cudaMemcpy(pool->dev_layer_ptrs, ptrs.data(), ptrs.size() * sizeof(void *),
+                   cudaMemcpyHostToDevice) != cudaSuccess) {
+        if (pool->dev_layer_ptrs)
+            cudaFree(pool->dev_layer_ptrs);
+        if (pool->owned)
+            cudaFree(pool->owned);
+        delete pool;
+        return CADKV_ERR_CUDA;
+    }
+    *out = pool;
+    return CADKV_OK;
+}
+
+int kv_pool_destroy(cadkv_pool *pool)
+{
+    if (!pool)
+        return CADKV_OK;
+    int rc = CADKV_OK;
+    if (pool->dev_layer_ptrs && cudaFree(pool->dev_layer_ptrs) != cudaSuccess)
+        rc = CADKV_ERR_CUDA;
+    if (pool->owned && cudaFree(pool->owned) != cudaSuccess)
+        rc = CADKV_ERR_CUDA;
+    delete pool;
+    return rc;
+}
+
+int kv_pool_layer(const cadkv_pool *pool, int layer, void **k_pages, void **v_pages)
+{
+    if (!pool || layer < 0 || layer >= pool->num_layers)
+        return CADKV_ERR_INVALID;
+    if (k_pages)
+        *k_pages = pool->k[layer];
+    if (v_pages)
+        *v_pages = pool->v[layer];
+    return CADKV_OK;
+}
+
+int kv_pool_geometry(const cadkv_pool *pool, int *num_layers, int *num_pages, int *page_size,
+                     int *num_kv_heads, int *head_dim)
+{
+    if (!pool)
+        return CADKV_ERR_INVALID;
+    if (num_layers)
+        *num_layers = pool->num_layers;
+    if (num_pages)
+        *num_pages = pool->num_pages;
+    if (page_size)
+        *page_size = pool->page_size;
+    if (num_kv_heads)
+        *num_kv_heads = pool->num_kv_heads;
+    if (head_dim)
+        *head_dim = pool->head_dim;
+    return CADKV_OK;
+}
+
+size_t decode_attention_workspace_size(int batch, int num_q_heads, int num_kv_heads,
+                                       int head_dim, int max_pages)
+{
+    const DecodeShape s{batch, num_q_heads, num_kv_heads, head_dim, kPageSize, 1, max_pages};
+    if (check_decode_shape(s) != CADKV_OK)
+        return 0;
+    const int sms = device_sms();
+    if (sms < 0)
+        return 0;
+    return decode_workspace_layout(batch, num_kv_heads, num_q_heads / num_kv_heads, head_dim, sms)
+        .total;
+}
+
+int decode_attention_plan(const int32_t *context_lens, void *out, float *lse, int batch,
+                          int num_q_heads, int num_kv_heads, int head_dim, int max_pages,
+                          int slice_pages, void *workspace, size_t workspace_bytes,
+                          cadkv_stream_t stream)
+{
+    const DecodeShape s{batch, num_q_heads, num_kv_heads, head_dim, kPageSize, 1, max_pages};
+    return plan_impl(context_lens, out, lse, s, slice_pages, workspace, workspace_bytes,
+                     reinterpret_cast<cudaStream_t>(stream));
+}
+
+int decode_attention_run(const void *q, const void *k_pages, const void *v_pages,
+                         const int32_t *block_table, const int32_t *context_lens, void *out,
+                         float *lse, int batch, int num_q_heads, int num_kv_heads, int head_dim,
+                         int page_size, int num_pages, int max_pages, void *workspace,
+                         size_t workspace_bytes, cadkv_stream_t stream)
+{
+    const DecodeShape s{batch, num_q_heads, num_kv_heads, head_dim, page_size, num_pages, max_pages};
+    return run_impl(q, k_pages, v_pages, block_table, context_lens, out, lse, s, workspace,
+                    workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int decode_attention_split(const void *q, const void *k_pages, const void *v_pages,
+                           const int32_t *block_table, const int32_t *context_lens, void *out,
+                           float *lse, int batch, int num_q_heads, int num_kv_heads,
+                           int head_dim, int page_size, int num_pages, int max_pages,
+                           int slice_pages, void *workspace, size_t workspace_bytes,
+                           cadkv_stream_t stream)
+{
+    const DecodeShape s{batch, num_q_heads, num_kv_heads, head_dim, page_size, num_pages, max_pages};
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    // Validate everything the run needs before launching the planner.
+    int rc = check_decode_shape(s);
+    if (rc != CADKV_OK)
+        return rc;
+    if (batch == 0)
+        return CADKV_OK;
+    rc = check_run_args(q, k_pages, v_pages, block_table, context_lens, out, lse, s);
+    if (rc != CADKV_OK)
+        return rc;
+    rc = plan_impl(context_lens, out, lse, s, slice_pages, workspace, workspace_bytes, st);
+    if (rc != CADKV_OK)
+        return rc;
+    return run_impl(q, k_pages, v_pages, block_table, context_lens, out, lse, s, workspace,
+                    workspace_bytes, st);
+}
+
+int decode_attention(const void *q, const void *k_pages, const void *v_pages,
+                     const int32_t *block_table, const int32_t *context_lens, void *out,
+                     float *lse, int batch, int num_q_heads, int num_kv_heads, int head_dim,
+                     int page_size, int num_pages, int max_pages, void *workspace,
+                     size_t workspace_bytes, cadkv_stream_t stream)
+{
+    return decode_attention_split(q, k_pages, v_pages, block_table, context_lens, out, lse,
+                                  batch, num_q_heads, num_kv_heads, head_dim, page_size,
+                                  num_pages, max_pages, 0, workspace, workspace_bytes, stream);
+}
+
+int decode_attention_status(const void *workspace, cadkv_stream_t stream)
+{
+    return read_status(workspace, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t kv_prefix_stage_workspace_size(int batch)
+{
+    if (batch < 0)
+        return 0;
+    return stage_workspace_layout(batch).total;
+}
+
+int kv_prefix_stage(const cadkv_pool *pool, const int32_t *block_table, int max_pages,
+                    const int32_t *context_lens, int batch, int layer_begin, int layer_end,
+                    void *dst, const int64_t *dst_offsets, void *workspace,
+                    size_t workspace_bytes, cadkv_stream_t stream)
+{
+    return stage_impl(pool, block_table, max_pages, context_lens, batch, layer_begin, layer_end,
+                      dst, dst_offsets, workspace, workspace_bytes,
+                      reinterpret_cast<cudaStream_t>(stream), 0);
+}
+
+int kv_prefix_load(const cadkv_pool *pool, const int32_t *block_table, int max_pages,
+                   const int32_t *context_lens, int batch, int layer_begin, int layer_end,
+                   const void *src, const int64_t *src_offsets, void *workspace,
+                   size_t workspace_bytes, cadkv_stream_t stream)
+{
+    return stage_impl(pool, block_table, max_pages, context_lens, batch, layer_begin, layer_end,
+                      src, src_offsets, workspace, workspace_bytes,
+                      reinterpret_cast<cudaStream_t>(stream), 1);
+}
+
+int kv_prefix_stage_status(const void *workspace, cadkv_stream_t stream)
+{
+    return read_status(workspace, reinterpret_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"

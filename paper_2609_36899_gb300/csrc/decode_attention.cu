@@ -1,0 +1,708 @@
+// decode_attention.cu -- batched paged-KV decode attention for sm_103a.
+//
+// One decode step of scaled dot-product attention (one query token per
+// trajectory) over a paged KV cache.  The decode step is the memory-bound
+// phase the paper's scheduler reshapes (Sec. 2.3, Sec. 3.1); attention and the
+// paged cache themselves come from the paper's inference backend (Sec. 5).
+//
+// Design (GB300-first):
+//  * Work = the flattened sequence of (trajectory b, KV head g, page j)
+//    "page-heads", ordered b-major.  A planner kernel computes the page prefix
+//    sum over trajectories; the sequence is cut into T equal slices, which a
+//    persistent grid (one CTA per SM) pulls with an atomic counter.  Equal
+//    slices balance HBM bytes, not trajectories, so a few 128K-token tails and
+//    hundreds of 2K-token trajectories both keep every SM streaming.
+//  * Inside a CTA one producer warp issues TMA copies (cp.async.bulk.tensor,
+//    128-byte swizzle) of each page-head's K and V block (16 tokens x D bf16,
+//    contiguous in the head-major pool) into a ring of shared-memory stages
+//    guarded by mbarriers, plus a 1-D bulk copy of the G query rows of every
+//    new segment.  Each KV page is read from HBM exactly once per KV head:
+//    all G query heads of the group share it (grouped-query attention).
+//  * Four consumer warps take pages round-robin.  Per page a warp computes
+//    S^T = K Q^T with mma.sync m16n8k16 (16 tokens x 8 query heads), runs the
+//    online softmax in registers (warp shuffles for the per-head max), turns
+//    P^T into the B operand with movmatrix, and accumulates O^T += V^T P^T.
+//  * At the end of a segment the warps merge their (m, l, O) in shared memory.
+//    A trajectory-head that lies inside one slice is written straight to
+//    `out`; otherwise the slice writes a partial (o, log2-sum-exp) and the CTA
+//    that delivers a unit's last partial merges all of them in slice order
+//    (deterministic), so no separate merge kernel runs.
+//  * Every wait is bounded (kWaitLimitNs); on timeout the kernel records
+//    CADKV_ERR_TIMEOUT, drains its own copies and returns.
+#include <cfloat>
+#include <cmath>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace cadkv {
+
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr float kLn2 = 0.6931471805599453f;
+
+__host__ __device__ constexpr size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// ------------------------------------------------------------------ planner
+
+__global__ void __launch_bounds__(1024, 1) plan_kernel(const PlanParams p)
+{
+    __shared__ long long warp_sums[32];
+    __shared__ long long carry_s;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int max_len = p.max_pages * kPageSize;
+    if (tid == 0) {
+        p.hdr->status = 0;
+        carry_s = 0;
+    }
+    __syncthreads();
+
+    for (int base = 0; base < p.batch; base += 1024) {
+        const int b = base + tid;
+        long long pages = 0;
+        if (b < p.batch) {
+            int n = p.context_lens[b];
+            if (n < 0 || n > max_len) {
+                record_status(&p.hdr->status, CADKV_ERR_SHAPE);
+                n = 0;
+            }
+            pages = (n + kPageSize - 1) / kPageSize;
+            if (n == 0) {  // empty trajectory: out = 0, lse = -inf
+                uint4 *row = reinterpret_cast<uint4 *>(p.out + (size_t)b * p.num_q_heads * p.head_dim);
+                const int vecs = p.num_q_heads * p.head_dim / 8;
+                for (int v = 0; v < vecs; ++v)
+                    row[v] = make_uint4(0, 0, 0, 0);
+                if (p.lse)
+                    for (int h = 0; h < p.num_q_heads; ++h)
+                        p.lse[(size_t)b * p.num_q_heads + h] = -INFINITY;
+            }
+        }
+        // block-wide inclusive scan of `pages`
+        long long v = pages;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            long long u = __shfl_up_sync(kFull, v, o);
+            if (lane >= o)
+                v += u;
+        }
+        if (lane == 31)
+            warp_sums[warp] = v;
+        __syncthreads();
+        if (warp == 0) {
+            long long w = warp_sums[lane];
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                long long u = __shfl_up_sync(kFull, w, o);
+                if (lane >= o)
+                    w += u;
+            }
+            warp_sums[lane] = w;  // inclusive over warps
+        }
+        __syncthreads();
+        const long long carry = carry_s;
+        const long long incl = carry + v + (warp > 0 ? warp_sums[warp - 1] : 0);
+        if (b < p.batch)
+            p.page_prefix[b] = incl - pages;
+        __syncthreads();
+        if (tid == 1023)
+            carry_s = incl;
+        __syncthreads();
+    }
+    for (int i = tid; i < p.batch * p.num_kv_heads; i += 1024)
+        p.unit_counter[i] = 0;
+    if (tid == 0) {
+        const long long total = carry_s;
+        p.page_prefix[p.batch] = total;
+        const long long W = total * p.num_kv_heads;
+        const long long unit = p.slice_pages > 0 ? p.slice_pages : kMinSlicePages;
+        long long T = (W + unit - 1) / unit;
+        if (T > p.slice_cap)
+            T = p.slice_cap;
+        if (T < 1)
+            T = 1;
+        p.hdr->total_work = W;
+        p.hdr->num_slices = (int)T;
+        p.hdr->slice_counter = 0;
+    }
+}
+
+// ------------------------------------------------------------------ attention
+
+struct SegDesc {
+    int b, kvh, page_begin, num_pages;  // num_pages < 0: no more work
+    int n, slot, count, unit;
+    int first, pad[3];
+};
+
+template <int D>
+struct AttnConfig {
+    static constexpr int kStages = D == 128 ? 20 : 28;
+    static constexpr int kBoxes = D / 64;                    // 64-element (128 B) TMA boxes per row
+    static constexpr int kBoxBytes = kPageSize * 128;        // 16 rows x 128 B
+    static constexpr int kKBytes = kBoxes * kBoxBytes;       // one page-head of K
+    static constexpr int kStageBytes = 2 * kKBytes;          // K + V
+    static constexpr int kQBytes = kMaxGroup * D * 2;        // one segment's query rows (padded)
+    static constexpr int kMergeStride = D + 4;               // floats per merge row (bank spread)
+    static constexpr size_t kStagesOff = 0;
+    static constexpr size_t kQOff = kStagesOff + (size_t)kStages * kStageBytes;
+    static constexpr size_t kMergeOOff = kQOff + (size_t)kSegRing * kQBytes;
+    static constexpr size_t kMergeMLOff =
+        kMergeOOff + (size_t)kNumConsumerWarps * kMaxGroup * kMergeStride * 4;
+    static constexpr size_t kDescOff = kMergeMLOff + (size_t)kNumConsumerWarps * kMaxGroup * 2 * 4;
+    static constexpr size_t kBarOff = align_up(kDescOff + (size_t)kSegRing * sizeof(SegDesc), 8);
+    static constexpr int kNumBars = 2 * kStages + 2 * kSegRing + 1;
+    static constexpr size_t kFlagOff = kBarOff + (size_t)kNumBars * 8;
+    static constexpr size_t kBytes = kFlagOff + 16 + 1024;  // + slack for 1024-B alignment
+};
+
+// Largest b in [0, batch) with prefix[b] <= v, given prefix non-decreasing,
+// prefix[0] = 0 <= v < prefix[batch].  Whole warp cooperates (32-way search).
+__device__ __forceinline__ int warp_find_trajectory(const long long *prefix, int batch,
+                                                    long long v, int lane)
+{
+    int lo = 0, hi = batch - 1;
+    while (lo < hi) {
+        const int span = hi - lo + 1;
+        const int step = (span + 31) / 32;
+        const int idx = lo + lane * step;
+        const bool pred = idx <= hi && prefix[idx] <= v;
+        const unsigned ballot = __ballot_sync(kFull, pred);
+        const int last = 31 - __clz(ballot);  // lane 0 always true (prefix[lo] <= v)
+        lo = lo + last * step;
+        hi = min(hi, lo + step - 1);
+    }
+    return lo;
+}
+
+__device__ __forceinline__ long long slice_begin(long long s, long long W, long long T)
+{
+    return s * W / T;
+}
+
+// Index of the slice containing flattened position x.
+__device__ __forceinline__ int slice_of(long long x, long long W, long long T)
+{
+    return (int)(((x + 1) * T + W - 1) / W - 1);
+}
+
+// All 128 consumer threads arrive and wait; bounded, abort-aware.
+__device__ __forceinline__ bool consumer_sync(uint64_t *bar, uint32_t &phase, volatile int *abort)
+{
+    mbar_arrive(bar);
+    const bool ok = mbar_wait(bar, phase, abort);
+    phase ^= 1u;
+    return __all_sync(kFull, ok);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kAttnThreads, 1)
+    decode_attention_kernel(const AttnParams p, const __grid_constant__ CUtensorMap kmap,
+                            const __grid_constant__ CUtensorMap vmap)
+{
+    using C = AttnConfig<D>;
+    constexpr int S = C::kStages;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(align_up(reinterpret_cast<size_t>(smem_raw), 1024));
+    uint8_t *stages = smem + C::kStagesOff;
+    __nv_bfloat16 *qbuf = reinterpret_cast<__nv_bfloat16 *>(smem + C::kQOff);
+    float *merge_o = reinterpret_cast<float *>(smem + C::kMergeOOff);
+    float *merge_m = reinterpret_cast<float *>(smem + C::kMergeMLOff);
+    float *merge_l = merge_m + kNumConsumerWarps * kMaxGroup;
+    SegDesc *desc = reinterpret_cast<SegDesc *>(smem + C::kDescOff);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kBarOff);
+    uint64_t *full_bar = bars;
+    uint64_t *empty_bar = bars + S;
+    uint64_t *seg_full = bars + 2 * S;
+    uint64_t *seg_empty = seg_full + kSegRing;
+    uint64_t *cons_bar = seg_empty + kSegRing;
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + C::kFlagOff);
+    volatile int *is_last_flag = abort_flag + 1;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int G = p.group;
+    const int Hkv = p.num_kv_heads;
+
+    if (tid == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], 1);
+        }
+        for (int r = 0; r < kSegRing; ++r) {
+            mbar_init(&seg_full[r], 1);
+            mbar_init(&seg_empty[r], kNumConsumerWarps);
+        }
+        mbar_init(cons_bar, kNumConsumerWarps * 32);
+        *abort_flag = 0;
+        *is_last_flag = 0;
+        fence_mbarrier_init();
+    }
+    // Query rows G..7 of every segment slot stay zero (TMA writes rows < G).
+    for (int i = tid; i < kSegRing * kMaxGroup * D / 8; i += kAttnThreads) {
+        const int row = (i / (D / 8)) % kMaxGroup;
+        if (row >= G)
+            reinterpret_cast<uint4 *>(qbuf)[i] = make_uint4(0, 0, 0, 0);
+    }
+    __syncthreads();
+
+    const long long W = p.hdr->total_work;
+    const int T = p.hdr->num_slices;
+
+    if (warp == kNumConsumerWarps) {
+        // ============================ producer warp ============================
+        if (lane == 0) {
+            prefetch_tensor_map(&kmap);
+            prefetch_tensor_map(&vmap);
+        }
+        const uint64_t policy = l2_evict_first_policy();
+        const uint32_t q_bytes = (uint32_t)(G * D * 2);
+        uint32_t kp = 0;  // page-heads issued
+        uint32_t sp = 0;  // segments issued
+        bool ok = true;
+        while (ok) {
+            int slice = 0;
+            if (lane == 0)
+                slice = atomicAdd(&p.hdr->slice_counter, 1);
+            slice = __shfl_sync(kFull, slice, 0);
+            if (slice >= T)
+                break;
+            const long long s0 = slice_begin(slice, W, T), s1 = slice_begin(slice + 1, W, T);
+            if (s0 >= s1)
+                continue;
+            int b = warp_find_trajectory(p.page_prefix, p.batch, s0 / Hkv, lane);
+            long long x = s0;
+            while (x < s1) {
+                const long long pb0 = p.page_prefix[b], pb1 = p.page_prefix[b + 1];
+                if (x >= pb1 * Hkv) {
+                    ++b;
+                    continue;
+                }
+                const long long pages_b = pb1 - pb0;
+                const long long base = pb0 * Hkv;
+                const int kvh = (int)((x - base) / pages_b);
+                const long long us = base + kvh * pages_b, ue = us + pages_b;
+                const int j0 = (int)(x - us);
+                const long long se = ue < s1 ? ue : s1;
+                const int npg = (int)(se - x);
+                const int first = slice_of(us, W, T), last = slice_of(ue - 1, W, T);
+                const int count = last - first + 1;
+                const int unit = b * Hkv + kvh;
+
+                const uint32_t r = sp % kSegRing;
+                if (sp >= kSegRing) {
+                    ok = mbar_wait(&seg_empty[r], ((sp / kSegRing) + 1) & 1, abort_flag);
+                    ok = __all_sync(kFull, ok);
+                    if (!ok)
+                        break;
+                }
+                if (lane == 0) {
+                    int n = p.context_lens[b];
+                    if (n > (int)(pages_b * kPageSize))
+                        n = (int)(pages_b * kPageSize);
+                    SegDesc d;
+                    d.b = b;
+                    d.kvh = kvh;
+                    d.page_begin = j0;
+                    d.num_pages = npg;
+                    d.n = n;
+                    d.slot = count == 1 ? -1 : unit + slice;
+                    d.count = count;
+                    d.unit = unit;
+                    d.first = first;
+                    desc[r] = d;
+                    mbar_arrive_expect_tx(&seg_full[r], q_bytes);
+                    bulk_load(qbuf + (size_t)r * kMaxGroup * D,
+                              p.q + ((size_t)b * p.num_q_heads + (size_t)kvh * G) * D, q_bytes,
+                              &seg_full[r]);
+                }
+                ++sp;
+
+                const int *bt_row = p.block_table + (size_t)b * p.max_pages + j0;
+                for (int c = 0; c < npg && ok; c += 32) {
+                    int phys = 0;
+                    if (c + lane < npg) {
+                        phys = bt_row[c + lane];
+                        if (phys < 0 || phys >= p.num_pages) {
+                            record_status(&p.hdr->status, CADKV_ERR_OOB);
+                            phys = 0;
+                        }
+                    }
+                    const int cnt = min(32, npg - c);
+                    for (int i = 0; i < cnt; ++i) {
+                        const int ph = __shfl_sync(kFull, phys, i);
+                        const uint32_t st = kp % S;
+                        if (kp >= (uint32_t)S) {
+                            ok = mbar_wait(&empty_bar[st], ((kp / S) + 1) & 1, abort_flag);
+                            ok = __all_sync(kFull, ok);
+                            if (!ok)
+                                break;
+                        }
+                        if (lane == 0) {
+                            uint8_t *kdst = stages + (size_t)st * C::kStageBytes;
+                            uint8_t *vdst = kdst + C::kKBytes;
+                            const int y = (ph * Hkv + kvh) * kPageSize;
+                            mbar_arrive_expect_tx(&full_bar[st], C::kStageBytes);
+#pragma unroll
+                            for (int bx = 0; bx < C::kBoxes; ++bx) {
+                                tma_load_2d(kdst + bx * C::kBoxBytes, &kmap, bx * 64, y, &full_bar[st], policy);
+                                tma_load_2d(vdst + bx * C::kBoxBytes, &vmap, bx * 64, y, &full_bar[st], policy);
+                            }
+                        }
+                        ++kp;
+                    }
+                }
+                if (!ok)
+                    break;
+                x = se;
+            }
+        }
+        // End-of-work sentinel.
+        if (ok) {
+            const uint32_t r = sp % kSegRing;
+            if (sp >= kSegRing) {
+                ok = mbar_wait(&seg_empty[r], ((sp / kSegRing) + 1) & 1, abort_flag);
+                ok = __all_sync(kFull, ok);
+            }
+            if (ok && lane == 0) {
+                desc[r].num_pages = -1;
+                mbar_arrive(&seg_full[r]);
+            }
+        }
+        if (!ok && lane == 0) {
+            *abort_flag = 1;
+            record_status(&p.hdr->status, CADKV_ERR_TIMEOUT);
+        }
+        // Drain: every copy this warp issued must land before the CTA exits.
+        if (lane == 0) {
+            const uint32_t k_lo = kp > (uint32_t)S ? kp - S : 0;
+            for (uint32_t k = k_lo; k < kp; ++k) {
+                volatile int never = 0;
+                mbar_wait(&full_bar[k % S], (k / S) & 1, &never);
+            }
+            const uint32_t s_lo = sp > (uint32_t)kSegRing ? sp - kSegRing : 0;
+            for (uint32_t s = s_lo; s < sp; ++s) {
+                volatile int never = 0;
+                mbar_wait(&seg_full[s % kSegRing], (s / kSegRing) & 1, &never);
+            }
+        }
+        return;
+    }
+
+    // ================================ consumer warps ================================
+    const int g = lane >> 2, t = lane & 3;          // mma fragment coordinates
+    const int mi = lane >> 3, rr = lane & 7;        // ldmatrix: matrix index, row in matrix
+    const int ct = tid;                             // consumer thread 0..127
+    uint32_t k = 0, sc = 0, cphase = 0;
+    bool ok = true;
+
+    for (;;) {
+        const uint32_t r = sc % kSegRing;
+        ok = __all_sync(kFull, mbar_wait(&seg_full[r], (sc / kSegRing) & 1, abort_flag));
+        if (!ok)
+            break;
+        const SegDesc d = desc[r];
+        if (d.num_pages < 0)
+            break;
+
+        // B operand of S^T = K Q^T: b0 = Q[g][16kk + 2t .. +1], b1 = Q[g][16kk + 8 + 2t .. +1]
+        uint32_t qf[D / 16][2];
+        {
+            const __nv_bfloat16 *qs = qbuf + (size_t)r * kMaxGroup * D + g * D + 2 * t;
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+                qf[kk][0] = *reinterpret_cast<const uint32_t *>(qs + 16 * kk);
+                qf[kk][1] = *reinterpret_cast<const uint32_t *>(qs + 16 * kk + 8);
+            }
+        }
+        __syncwarp();
+        if (lane == 0)
+            mbar_arrive(&seg_empty[r]);
+        ++sc;
+
+        float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+        float o[D / 16][4];
+#pragma unroll
+        for (int mt = 0; mt < D / 16; ++mt)
+            o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+
+        const int npg = d.num_pages;
+        const int i0 = (int)((warp + kNumConsumerWarps - (int)(k % kNumConsumerWarps)) % kNumConsumerWarps);
+        for (int i = i0; i < npg; i += kNumConsumerWarps) {
+            const uint32_t kk_idx = k + i;
+            const uint32_t st = kk_idx % S;
+            ok = __all_sync(kFull, mbar_wait(&full_bar[st], (kk_idx / S) & 1, abort_flag));
+            if (!ok)
+                break;
+            const uint32_t kbase = smem_addr(stages + (size_t)st * C::kStageBytes);
+            const uint32_t vbase = kbase + C::kKBytes;
+            const int valid = min(kPageSize, d.n - (d.page_begin + i) * kPageSize);
+
+            // ---- S^T (16 tokens x 8 heads) = K (16 x D) . Q^T (D x 8)
+            float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
+            {
+                const int row = (mi & 1) * 8 + rr;
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const int chunk = 2 * kk + (mi >> 1);
+                    const uint32_t addr = kbase + (chunk >> 3) * C::kBoxBytes + row * 128 +
+                                          (((chunk & 7) ^ rr) << 4);
+                    uint32_t a0, a1, a2, a3;
+                    ldmatrix_x4(addr, a0, a1, a2, a3);
+                    if (kk & 1)
+                        mma_bf16_m16n8k16(sb, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
+                    else
+                        mma_bf16_m16n8k16(sa, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
+                }
+            }
+            // s[0]: (token g, head 2t)  s[1]: (g, 2t+1)  s[2]: (g+8, 2t)  s[3]: (g+8, 2t+1)
+            float s[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                s[e] = (sa[e] + sb[e]) * p.scale_log2;
+            if (valid < kPageSize) {
+                if (g >= valid) {
+                    s[0] = -INFINITY;
+                    s[1] = -INFINITY;
+                }
+                if (g + 8 >= valid) {
+                    s[2] = -INFINITY;
+                    s[3] = -INFINITY;
+                }
+            }
+            float mx0 = fmaxf(s[0], s[2]), mx1 = fmaxf(s[1], s[3]);
+#pragma unroll
+            for (int off = 4; off < 32; off <<= 1) {
+                mx0 = fmaxf(mx0, __shfl_xor_sync(kFull, mx0, off));
+                mx1 = fmaxf(mx1, __shfl_xor_sync(kFull, mx1, off));
+            }
+            const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+            const float alpha0 = exp2_approx(m0 - mn0), alpha1 = exp2_approx(m1 - mn1);
+            m0 = mn0;
+            m1 = mn1;
+            const float p0 = exp2_approx(s[0] - mn0), p1 = exp2_approx(s[1] - mn1);
+            const float p2 = exp2_approx(s[2] - mn0), p3 = exp2_approx(s[3] - mn1);
+            l0 = l0 * alpha0 + (p0 + p2);
+            l1 = l1 * alpha1 + (p1 + p3);
+#pragma unroll
+            for (int mt = 0; mt < D / 16; ++mt) {
+                o[mt][0] *= alpha0;
+                o[mt][1] *= alpha1;
+                o[mt][2] *= alpha0;
+                o[mt][3] *= alpha1;
+            }
+            // P^T as the B operand: transpose the two 8x8 (token x head) blocks.
+            const uint32_t pb0 = movmatrix_trans(pack_bf16x2(p0, p1));
+            const uint32_t pb1 = movmatrix_trans(pack_bf16x2(p2, p3));
+            uint32_t mask_lo = 0xffffffffu, mask_hi = 0xffffffffu;
+            if (valid < kPageSize) {  // zero value rows past n (they may hold NaN)
+                mask_lo = (2 * t < valid ? 0x0000ffffu : 0u) | (2 * t + 1 < valid ? 0xffff0000u : 0u);
+                mask_hi = (2 * t + 8 < valid ? 0x0000ffffu : 0u) | (2 * t + 9 < valid ? 0xffff0000u : 0u);
+            }
+            // ---- O^T (D x 8) += V^T (D x 16 tokens) . P^T (16 x 8)
+            {
+                const int row = (mi >> 1) * 8 + rr;
+#pragma unroll
+                for (int mt = 0; mt < D / 16; ++mt) {
+                    const int chunk = 2 * mt + (mi & 1);
+                    const uint32_t addr = vbase + (chunk >> 3) * C::kBoxBytes + row * 128 +
+                                          (((chunk & 7) ^ rr) << 4);
+                    uint32_t a0, a1, a2, a3;
+                    ldmatrix_x4_trans(addr, a0, a1, a2, a3);
+                    a0 &= mask_lo;
+                    a1 &= mask_lo;
+                    a2 &= mask_hi;
+                    a3 &= mask_hi;
+                    mma_bf16_m16n8k16(o[mt], a0, a1, a2, a3, pb0, pb1);
+                }
+            }
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&empty_bar[st]);
+        }
+        if (!ok)
+            break;
+        k += npg;
+
+        // ---- per-warp totals: l summed over the 8 lanes sharing t
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) {
+            l0 += __shfl_xor_sync(kFull, l0, off);
+            l1 += __shfl_xor_sync(kFull, l1, off);
+        }
+        {
+            float *mo = merge_o + (size_t)warp * kMaxGroup * C::kMergeStride;
+#pragma unroll
+            for (int mt = 0; mt < D / 16; ++mt) {
+                mo[(2 * t) * C::kMergeStride + 16 * mt + g] = o[mt][0];
+                mo[(2 * t + 1) * C::kMergeStride + 16 * mt + g] = o[mt][1];
+                mo[(2 * t) * C::kMergeStride + 16 * mt + g + 8] = o[mt][2];
+                mo[(2 * t + 1) * C::kMergeStride + 16 * mt + g + 8] = o[mt][3];
+            }
+            if (g == 0) {
+                merge_m[warp * kMaxGroup + 2 * t] = m0;
+                merge_m[warp * kMaxGroup + 2 * t + 1] = m1;
+                merge_l[warp * kMaxGroup + 2 * t] = l0;
+                merge_l[warp * kMaxGroup + 2 * t + 1] = l1;
+            }
+        }
+        ok = consumer_sync(cons_bar, cphase, abort_flag);
+        if (!ok)
+            break;
+
+        // ---- combine the warps; write the result or this slice's partial
+        const bool partial = d.slot >= 0;
+        const int q_head0 = d.kvh * G;
+        for (int it = ct; it < G * (D / 8); it += kNumConsumerWarps * 32) {
+            const int h = it / (D / 8), d0 = (it % (D / 8)) * 8;
+            float M = -INFINITY;
+#pragma unroll
+            for (int w = 0; w < kNumConsumerWarps; ++w)
+                M = fmaxf(M, merge_m[w * kMaxGroup + h]);
+            float L = 0.f, acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int w = 0; w < kNumConsumerWarps; ++w) {
+                const float sc_w = exp2_approx(merge_m[w * kMaxGroup + h] - M);
+                L += merge_l[w * kMaxGroup + h] * sc_w;
+                const float *src = merge_o + ((size_t)w * kMaxGroup + h) * C::kMergeStride + d0;
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    acc[e] += src[e] * sc_w;
+            }
+            const float inv = 1.f / L;
+            const float lse2 = M + __log2f(L);
+            if (!partial) {
+                uint4 packed;
+                packed.x = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+                packed.y = pack_bf16x2(acc[2] * inv, acc[3] * inv);
+                packed.z = pack_bf16x2(acc[4] * inv, acc[5] * inv);
+                packed.w = pack_bf16x2(acc[6] * inv, acc[7] * inv);
+                const size_t row = (size_t)d.b * p.num_q_heads + q_head0 + h;
+                *reinterpret_cast<uint4 *>(p.out + row * D + d0) = packed;
+                if (d0 == 0 && p.lse)
+                    p.lse[row] = lse2 * kLn2;
+            } else {
+                float4 *dst = reinterpret_cast<float4 *>(p.part_o + ((size_t)d.slot * G + h) * D + d0);
+                dst[0] = make_float4(acc[0] * inv, acc[1] * inv, acc[2] * inv, acc[3] * inv);
+                dst[1] = make_float4(acc[4] * inv, acc[5] * inv, acc[6] * inv, acc[7] * inv);
+                if (d0 == 0)
+                    p.part_lse[(size_t)d.slot * G + h] = lse2;
+            }
+        }
+        if (partial)
+            __threadfence();
+        ok = consumer_sync(cons_bar, cphase, abort_flag);
+        if (!ok)
+            break;
+        if (!partial)
+            continue;
+
+        // ---- the CTA that completes a unit merges its partials in slice order
+        if (ct == 0) {
+            const int old = atomicAdd(&p.unit_counter[d.unit], 1);
+            *is_last_flag = (old == d.count - 1) ? 1 : 0;
+        }
+        ok = consumer_sync(cons_bar, cphase, abort_flag);
+        if (!ok)
+            break;
+        if (*is_last_flag) {
+            __threadfence();
+            const int slot0 = d.unit + d.first;
+            for (int it = ct; it < G * (D / 8); it += kNumConsumerWarps * 32) {
+                const int h = it / (D / 8), d0 = (it % (D / 8)) * 8;
+                float M = -INFINITY;
+                for (int s2 = 0; s2 < d.count; ++s2)
+                    M = fmaxf(M, __ldcg(p.part_lse + (size_t)(slot0 + s2) * G + h));
+                float L = 0.f, acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                for (int s2 = 0; s2 < d.count; ++s2) {
+                    const size_t sl = (size_t)(slot0 + s2);
+                    const float w = exp2_approx(__ldcg(p.part_lse + sl * G + h) - M);
+                    L += w;
+                    const float4 *src = reinterpret_cast<const float4 *>(p.part_o + (sl * G + h) * D + d0);
+                    const float4 u0 = __ldcg(src), u1 = __ldcg(src + 1);
+                    acc[0] += w * u0.x;
+                    acc[1] += w * u0.y;
+                    acc[2] += w * u0.z;
+                    acc[3] += w * u0.w;
+                    acc[4] += w * u1.x;
+                    acc[5] += w * u1.y;
+                    acc[6] += w * u1.z;
+                    acc[7] += w * u1.w;
+                }
+                const float inv = 1.f / L;
+                uint4 packed;
+                packed.x = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+                packed.y = pack_bf16x2(acc[2] * inv, acc[3] * inv);
+                packed.z = pack_bf16x2(acc[4] * inv, acc[5] * inv);
+                packed.w = pack_bf16x2(acc[6] * inv, acc[7] * inv);
+                const size_t row = (size_t)d.b * p.num_q_heads + q_head0 + h;
+                *reinterpret_cast<uint4 *>(p.out + row * D + d0) = packed;
+                if (d0 == 0 && p.lse)
+                    p.lse[row] = (M + __log2f(L)) * kLn2;
+            }
+        }
+    }
+    if (!ok && lane == 0) {
+        *abort_flag = 1;
+        record_status(&p.hdr->status, CADKV_ERR_TIMEOUT);
+    }
+}
+
+template <int D>
+cudaError_t launch_attention_d(const AttnParams &p, const CUtensorMap &kmap,
+                               const CUtensorMap &vmap, int grid, cudaStream_t stream)
+{
+    static bool configured = false;
+    const size_t smem = AttnConfig<D>::kBytes;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(decode_attention_kernel<D>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess)
+            return e;
+        configured = true;
+    }
+    decode_attention_kernel<D><<<grid, kAttnThreads, smem, stream>>>(p, kmap, vmap);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+DecodeWorkspaceLayout decode_workspace_layout(int batch, int num_kv_heads, int group,
+                                              int head_dim, int num_sms)
+{
+    DecodeWorkspaceLayout L{};
+    L.slice_cap = num_sms * kSlicesPerCta;
+    L.capacity = batch * num_kv_heads + L.slice_cap;
+    size_t off = align_up(sizeof(WorkspaceHeader), kWorkspaceAlign);
+    L.page_prefix = off;
+    off = align_up(off + (size_t)(batch + 1) * sizeof(long long), kWorkspaceAlign);
+    L.unit_counter = off;
+    off = align_up(off + (size_t)batch * num_kv_heads * sizeof(int), kWorkspaceAlign);
+    L.part_lse = off;
+    off = align_up(off + (size_t)L.capacity * group * sizeof(float), kWorkspaceAlign);
+    L.part_o = off;
+    off = align_up(off + (size_t)L.capacity * group * head_dim * sizeof(float), kWorkspaceAlign);
+    L.total = off;
+    return L;
+}
+
+cudaError_t launch_plan(const PlanParams &p, cudaStream_t stream)
+{
+    plan_kernel<<<1, 1024, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+size_t attention_smem_bytes(int head_dim)
+{
+    return head_dim == 128 ? AttnConfig<128>::kBytes : AttnConfig<64>::kBytes;
+}
+
+cudaError_t launch_attention(const AttnParams &p, const CUtensorMap &kmap,
+                             const CUtensorMap &vmap, int head_dim, int grid,
+                             cudaStream_t stream)
+{
+    if (head_dim == 128)
+        return launch_attention_d<128>(p, kmap, vmap, grid, stream);
+    return launch_attention_d<64>(p, kmap, vmap, grid, stream);
+}
+
+}  // namespace cadkv

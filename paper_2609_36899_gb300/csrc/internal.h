@@ -1,0 +1,105 @@
+// internal.h -- types shared by the host launchers and the kernels.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "../../include/cadkv.h"
+
+namespace cadkv {
+
+constexpr int kPageSize = 16;      // tokens per KV page
+constexpr int kMaxGroup = 8;       // query heads per KV head handled by one tile
+constexpr int kNumConsumerWarps = 4;
+constexpr int kAttnThreads = (kNumConsumerWarps + 1) * 32;
+constexpr int kSegRing = 8;        // segment descriptors in flight per CTA
+constexpr int kSlicesPerCta = 4;   // dynamic work slices per persistent CTA
+constexpr int kMinSlicePages = 16; // auto slicing never cuts finer than this
+constexpr size_t kWorkspaceAlign = 256;
+
+// Header at the start of a decode-attention or staging workspace.
+struct alignas(64) WorkspaceHeader {
+    int status;            // first device-side error code, 0 = none
+    int slice_counter;     // next work slice to hand out
+    int num_slices;        // T: slices of the flattened work sequence
+    int pad0;
+    long long total_work;  // W: page-heads (decode) or copy units (staging)
+    long long pad1[5];
+};
+
+// Byte offsets of the decode-attention workspace regions.
+struct DecodeWorkspaceLayout {
+    size_t page_prefix;   // int64 [batch + 1]
+    size_t unit_counter;  // int32 [batch * Hkv]
+    size_t part_lse;      // fp32  [capacity][G]
+    size_t part_o;        // fp32  [capacity][G][D]
+    size_t total;
+    int capacity;         // partial slots = batch * Hkv + slice cap
+    int slice_cap;
+};
+
+DecodeWorkspaceLayout decode_workspace_layout(int batch, int num_kv_heads, int group,
+                                              int head_dim, int num_sms);
+
+struct PlanParams {
+    const int *context_lens;
+    __nv_bfloat16 *out;
+    float *lse;
+    WorkspaceHeader *hdr;
+    long long *page_prefix;
+    int *unit_counter;
+    int batch, num_q_heads, num_kv_heads, head_dim, max_pages;
+    int slice_cap;      // upper bound on slices (partial capacity)
+    int slice_pages;    // forced slice length in pages, 0 = automatic
+};
+
+struct AttnParams {
+    const __nv_bfloat16 *q;
+    const int *block_table;
+    const int *context_lens;
+    __nv_bfloat16 *out;
+    float *lse;
+    WorkspaceHeader *hdr;
+    const long long *page_prefix;
+    int *unit_counter;
+    float *part_lse;
+    float *part_o;
+    int batch, num_q_heads, num_kv_heads, group, max_pages, num_pages;
+    float scale_log2;  // log2(e) / sqrt(D)
+};
+
+cudaError_t launch_plan(const PlanParams &p, cudaStream_t stream);
+cudaError_t launch_attention(const AttnParams &p, const CUtensorMap &kmap,
+                             const CUtensorMap &vmap, int head_dim, int grid,
+                             cudaStream_t stream);
+size_t attention_smem_bytes(int head_dim);
+
+// ---------------------------------------------------------------- staging
+
+struct StageParams {
+    const void *const *layer_k;  // device array [num_layers] of K page pointers
+    const void *const *layer_v;  // device array [num_layers] of V page pointers
+    const int *block_table;
+    const int *context_lens;
+    void *rows;                  // staged rows (dst of stage, src of load)
+    const long long *row_offsets;  // nullable
+    WorkspaceHeader *hdr;
+    long long *page_prefix;      // [B + 1]
+    long long *token_prefix;     // [B + 1]
+    long long *unit_prefix;      // [B + 1]
+    int batch, max_pages, num_pages, num_kv_heads, head_dim;
+    int layer_begin, layer_end;
+    int to_pool;                 // 0: pool -> rows (stage), 1: rows -> pool (load)
+};
+
+struct StageWorkspaceLayout {
+    size_t page_prefix, token_prefix, unit_prefix, total;
+};
+StageWorkspaceLayout stage_workspace_layout(int batch);
+
+cudaError_t launch_stage(const StageParams &p, int num_sms, cudaStream_t stream);
+
+}  // namespace cadkv

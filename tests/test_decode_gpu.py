@@ -1,0 +1,233 @@
+"""GPU parity of decode attention (CUDA path through the C ABI) against the
+fp64 oracle, on the same bf16 inputs.
+
+Sizes: the tiny workload in full; the paced / long-tail / mixed workloads at
+reduced batch sizes with their length distributions (full oracle), and at
+their full sizes in the bench's launch configuration on sampled trajectories;
+plus ragged, empty, maximal and degenerate cases and the method's invariances.
+"""
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_36899_gb300 as cadkv
+from paper_2609_36899_gb300 import STATUS
+from paper_2609_36899_gb300.workloads import (LONG_TAIL, MIXED, PACED, TINY, DecodeBatch,
+                                              bf16_bits, make_decode_batch)
+from _gpu_util import (assert_close, device_tensors, gpu_decode, make_batch,
+                       oracle_decode, sampled_oracle)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2609_36899_gb300 import build
+    build.build()
+
+
+def test_tiny_workload_full():
+    batch = make_decode_batch(TINY, device="cpu")
+    out, lse = gpu_decode(batch)
+    ref, ref_lse = oracle_decode(batch)
+    assert_close(out, lse, ref, ref_lse, "tiny")
+
+
+@pytest.mark.parametrize("w,bsz", [(PACED, 24), (LONG_TAIL, 2), (MIXED, 40)],
+                         ids=["paced", "long_tail", "mixed"])
+def test_reduced_workloads_full_oracle(w, bsz):
+    batch = make_decode_batch(w, device="cpu", batch=bsz)
+    out, lse = gpu_decode(batch)
+    ref, ref_lse = oracle_decode(batch)
+    assert_close(out, lse, ref, ref_lse, w.name)
+
+
+@pytest.mark.parametrize("w", [PACED, LONG_TAIL, MIXED], ids=["paced", "long_tail", "mixed"])
+def test_full_size_sampled(w):
+    """Full-size batch generated on the GPU, every output row finite, and the
+    longest, the shortest and four random trajectories against the oracle."""
+    batch = make_decode_batch(w, device="cuda")
+    tensors = (batch.q, batch.k_pages, batch.v_pages,
+               torch.from_numpy(batch.block_table).cuda(),
+               torch.from_numpy(batch.context_lens).cuda())
+    out, lse = gpu_decode(batch, tensors=tensors)
+    assert torch.isfinite(out.float()).all()
+    assert torch.isfinite(lse).all()
+    lens = batch.context_lens
+    rng = np.random.Generator(np.random.PCG64(7))
+    sample = sorted(set([int(np.argmax(lens)), int(np.argmin(lens))]
+                        + [int(x) for x in rng.choice(len(lens), 4, replace=False)]))
+    ref, ref_lse = sampled_oracle(batch, sample)
+    idx = torch.tensor(sample, device="cuda")
+    assert_close(out[idx], lse[idx], ref, ref_lse, f"{w.name} sampled {sample}")
+    del batch, tensors
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("g,d", [(1, 64), (2, 128), (4, 64), (8, 128), (8, 64), (3, 128)])
+def test_edge_lengths(g, d):
+    lens = [0, 1, 2, 15, 16, 17, 31, 32, 33, 255, 256, 257, 1000]
+    hkv = 2
+    batch = make_batch(lens, g * hkv, hkv, d, seed=100 + g * 10 + d)
+    out, lse = gpu_decode(batch)
+    ref, ref_lse = oracle_decode(batch)
+    assert_close(out, lse, ref, ref_lse, f"G={g} D={d}")
+    assert torch.all(out[0] == 0)
+    assert torch.all(torch.isneginf(lse[0]))
+
+
+def test_all_trajectories_empty():
+    batch = make_batch([0, 0, 0], 8, 2, 128, seed=3)
+    out, lse = gpu_decode(batch)
+    assert torch.all(out == 0)
+    assert torch.all(torch.isneginf(lse))
+
+
+def test_single_long_trajectory_at_table_limit():
+    max_pages = 512
+    batch = make_batch([max_pages * 16], 8, 1, 128, seed=4, max_pages=max_pages)
+    out, lse = gpu_decode(batch)
+    ref, ref_lse = oracle_decode(batch)
+    assert_close(out, lse, ref, ref_lse, "n = 16 * max_pages")
+
+
+@pytest.mark.parametrize("slice_pages", [1, 2, 3, 7, 16, 64, 1000, 1 << 20])
+def test_split_count_invariance(slice_pages):
+    """Forcing the work-slice length (how many partials each trajectory-head is
+    split into, and where) stays within tolerance of the oracle."""
+    batch = make_batch([3, 40, 700, 1900, 17, 5000], 16, 2, 128, seed=5)
+    out, lse = gpu_decode(batch, slice_pages=slice_pages)
+    ref, ref_lse = oracle_decode(batch)
+    assert_close(out, lse, ref, ref_lse, f"slice_pages={slice_pages}")
+
+
+def test_page_permutation_is_bit_identical():
+    """Moving physical pages (same logical content) changes no output bit: the
+    work split depends only on lengths."""
+    batch = make_batch([100, 513, 37, 2048], 16, 2, 128, seed=6, extra_pages=9)
+    out1, lse1 = gpu_decode(batch)
+    rng = np.random.Generator(np.random.PCG64(60))
+    perm = rng.permutation(batch.num_pages)          # new physical index of page p
+    inv = np.argsort(perm)
+    k2 = batch.k_pages[torch.from_numpy(inv)]
+    v2 = batch.v_pages[torch.from_numpy(inv)]
+    table2 = np.where(batch.block_table >= 0, perm[np.maximum(batch.block_table, 0)], -1)
+    b2 = DecodeBatch(batch.workload, batch.context_lens, table2.astype(np.int32), batch.q,
+                     k2, v2)
+    out2, lse2 = gpu_decode(b2)
+    assert torch.equal(out1, out2)
+    assert torch.equal(lse1, lse2)
+
+
+def test_deterministic_across_calls():
+    batch = make_batch([4000, 9000, 123, 77777 // 16], 32, 8, 128, seed=7)
+    tensors = device_tensors(batch)
+    a = gpu_decode(batch, tensors=tensors)
+    b = gpu_decode(batch, tensors=tensors)
+    assert torch.equal(a[0], b[0]) and torch.equal(a[1], b[1])
+
+
+def test_batch_order_invariance():
+    batch = make_batch([5, 900, 60, 3000, 1], 8, 2, 64, seed=8)
+    out, lse = gpu_decode(batch)
+    order = np.array([3, 0, 4, 1, 2])
+    b2 = DecodeBatch(batch.workload, batch.context_lens[order], batch.block_table[order],
+                     batch.q[torch.from_numpy(order)], batch.k_pages, batch.v_pages)
+    out2, lse2 = gpu_decode(b2)
+    ref, ref_lse = oracle_decode(batch)
+    assert_close(out2, lse2, ref[order], ref_lse[order], "permuted batch")
+    assert_close(out[torch.from_numpy(order).cuda()], lse[torch.from_numpy(order).cuda()],
+                 ref[order], ref_lse[order], "original batch")
+
+
+def test_gqa_matches_replicated_mha():
+    batch = make_batch([300, 45], 8, 2, 128, seed=9, nan_tails=False)
+    out, lse = gpu_decode(batch)
+    k_r = batch.k_pages.repeat_interleave(4, dim=1)
+    v_r = batch.v_pages.repeat_interleave(4, dim=1)
+    mha = DecodeBatch(batch.workload, batch.context_lens, batch.block_table, batch.q, k_r, v_r)
+    out2, lse2 = gpu_decode(mha)
+    ref, ref_lse = oracle_decode(batch)
+    assert_close(out, lse, ref, ref_lse, "GQA")
+    assert_close(out2, lse2, ref, ref_lse, "replicated MHA")
+
+
+def test_closed_forms_on_gpu():
+    """q = 0 gives mean V and lse = ln n; n = 1 returns V exactly."""
+    batch = make_batch([1, 50, 333], 8, 2, 128, seed=10)
+    batch.q.zero_()
+    batch.q[0].normal_()          # trajectory 0 (n = 1) keeps a random query
+    out, lse = gpu_decode(batch)
+    v = batch.v_pages.float()
+    for b, n in enumerate(batch.context_lens):
+        rows = [v[batch.block_table[b, t // 16], :, t % 16, :] for t in range(int(n))]
+        vs = torch.stack(rows)                       # [n, Hkv, D]
+        for h in range(8):
+            if b == 0:
+                assert torch.equal(out[0, h].cpu(), batch.v_pages[batch.block_table[0, 0], h // 4, 0])
+            else:
+                mean = vs[:, h // 4].double().mean(0).numpy()
+                err = np.abs(out[b, h].float().cpu().numpy() - mean).max()
+                assert err <= 1e-2, err
+                assert abs(lse[b, h].item() - np.log(n)) <= 1e-3 * np.log(n)
+
+
+def test_lse_is_optional():
+    batch = make_batch([70, 5], 4, 1, 64, seed=11)
+    out1, _ = gpu_decode(batch)
+    out2, lse2 = gpu_decode(batch, want_lse=False)
+    assert lse2 is None
+    assert torch.equal(out1, out2)
+
+
+def test_plan_then_run_equals_single_call():
+    batch = make_batch([700, 12, 3300], 16, 2, 128, seed=12)
+    q, k, v, bt, cl = device_tensors(batch)
+    out, lse = cadkv.decode_attention(q, k, v, bt, cl)
+    out2 = torch.empty_like(out)
+    lse2 = torch.empty_like(lse)
+    ws = torch.empty(cadkv.decode_attention_workspace_size(3, 16, 2, 128, bt.shape[1]),
+                     dtype=torch.uint8, device="cuda")
+    cadkv.decode_attention_plan(q, k, v, bt, cl, out2, lse2, ws)
+    cadkv.decode_attention_run(q, k, v, bt, cl, out2, lse2, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(out, out2) and torch.equal(lse, lse2)
+    assert cadkv.decode_attention_status(ws) == 0
+
+
+def test_status_reports_bad_page_without_faulting():
+    batch = make_batch([40, 20], 4, 1, 64, seed=13, nan_tails=False)
+    q, k, v, bt, cl = device_tensors(batch)
+    bt[1, 0] = batch.num_pages + 5                   # outside the pool
+    ws = torch.empty(cadkv.decode_attention_workspace_size(2, 4, 1, 64, bt.shape[1]),
+                     dtype=torch.uint8, device="cuda")
+    out, lse = cadkv.decode_attention(q, k, v, bt, cl, workspace=ws)
+    assert cadkv.decode_attention_status(ws) == STATUS["CADKV_ERR_OOB"]
+    ref, ref_lse = oracle_decode(DecodeBatch(batch.workload, batch.context_lens[:1],
+                                             batch.block_table[:1], batch.q[:1],
+                                             batch.k_pages, batch.v_pages))
+    assert_close(out[:1], lse[:1], ref, ref_lse, "untouched trajectory")
+    # the next good call clears the status
+    bt[1, 0] = int(batch.block_table[1, 0])
+    cadkv.decode_attention(q, k, v, bt, cl, workspace=ws)
+    assert cadkv.decode_attention_status(ws) == 0
+
+
+def test_status_reports_length_beyond_table():
+    batch = make_batch([40, 20], 4, 1, 64, seed=14, nan_tails=False)
+    q, k, v, bt, cl = device_tensors(batch)
+    cl[1] = bt.shape[1] * 16 + 1
+    ws = torch.empty(cadkv.decode_attention_workspace_size(2, 4, 1, 64, bt.shape[1]),
+                     dtype=torch.uint8, device="cuda")
+    out, lse = cadkv.decode_attention(q, k, v, bt, cl, workspace=ws)
+    assert cadkv.decode_attention_status(ws) == STATUS["CADKV_ERR_SHAPE"]
+    assert torch.all(out[1] == 0) and torch.all(torch.isneginf(lse[1]))
+
+
+def test_workspace_too_small_is_rejected():
+    batch = make_batch([40], 4, 1, 64, seed=15)
+    q, k, v, bt, cl = device_tensors(batch)
+    ws = torch.empty(64, dtype=torch.uint8, device="cuda")
+    with pytest.raises(cadkv.CadkvError) as e:
+        cadkv.decode_attention(q, k, v, bt, cl, workspace=ws)
+    assert e.value.status == STATUS["CADKV_ERR_WORKSPACE"]
