@@ -47,7 +47,7 @@ METRIC = "decode-attention achieved HBM GB/s (% of 8 TB/s) and decode steps/s pe
 NOMINAL_HBM_GBS = 8000.0
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
-PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "decode_attention_mixed_b512.md")
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "decode_attention_kernel_paced_b256.md")
 STAGE_PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "prefix_stage_copy_64traj.md")
 KERNEL_SOURCE = os.path.join(ROOT, "paper_2609_36899_gb300", "csrc", "decode_attention.cu")
 STAGE_SOURCE = os.path.join(ROOT, "paper_2609_36899_gb300", "csrc", "prefix_stage.cu")
@@ -150,7 +150,8 @@ def dist_setup(args):
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if world > 1:
         import torch.distributed as dist
-        torch.cuda.set_device(local)
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
     elif torch.cuda.is_available():
         torch.cuda.set_device(0)
@@ -299,11 +300,12 @@ def e2e_loop(batch, tensors, steps, warmup, stream):
     return secs, h2d, d2h
 
 
-def bench_staging(device, reps, layers=2):
-    """Prefix staging of all 64 trajectories of the staging workload for
-    ``layers`` layers (the full 48-layer job does not fit in HBM next to its
-    destination; it runs as 48 / layers such chunks)."""
-    job = make_staging_job(STAGING)
+def bench_staging(device, reps, layers=2, batch=None):
+    """Prefix staging of the staging workload's trajectories (all 64, or the
+    first ``batch`` of the same draw) for ``layers`` layers (the full 48-layer
+    job does not fit in HBM next to its destination; it runs as 48 / layers
+    such chunks)."""
+    job = make_staging_job(STAGING, batch=batch)
     k_layers = [torch.empty((job.num_pages, 8, 16, 128), dtype=torch.bfloat16, device=device)
                 for _ in range(layers)]
     v_layers = [torch.empty_like(k_layers[0]) for _ in range(layers)]
@@ -345,7 +347,7 @@ def bench_staging(device, reps, layers=2):
                                    got[l, kv].view(torch.int16)))
     peak, kind = hbm_peak()
     gbs = moved / (ms * 1e-3) / 1e9
-    res = {"workload": f"{STAGING.name}: 64 trajectories, {layers} of 48 layers per call",
+    res = {"workload": f"{STAGING.name}: {len(lens)} trajectories, {layers} of 48 layers per call",
            "gbps_read_plus_write": round(gbs, 1), "ms_per_call": round(ms, 3),
            "bytes_per_call": moved, "launches_per_call": 2, "status": status,
            "bit_exact_spot_check": ok,
@@ -403,7 +405,12 @@ def main():
     ap.add_argument("--steps", type=int, default=400)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=sorted(DECODE_WORKLOADS), default="mixed")
+    ap.add_argument("--workload", choices=sorted(DECODE_WORKLOADS) + ["staging"],
+                    default="mixed",
+                    help="decode workload of the headline line, or 'staging' to time "
+                         "only prefix staging")
+    ap.add_argument("--staging-layers", type=int, default=2)
+    ap.add_argument("--staging-batch", type=int, default=None)
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target oracle time of the cpu_baseline sample")
     ap.add_argument("--reference-seconds", type=float, default=90.0,
@@ -421,6 +428,12 @@ def main():
 
     pkg_build.build()
     device = torch.device("cuda", torch.cuda.current_device())
+    if args.workload == "staging":
+        res = bench_staging(device, reps=args.steps, layers=args.staging_layers,
+                            batch=args.staging_batch)
+        if rank == 0:
+            print(json.dumps(res), flush=True)
+        return
     w = DECODE_WORKLOADS[args.workload]
     batch = make_decode_batch(w, device=device, seed=w.seed + rank)
     tensors = _tensors(batch, device)
@@ -504,7 +517,7 @@ def main():
     del batch, tensors
     torch.cuda.empty_cache()
     if rank == 0 and not args.no_extras:
-        line["staging"] = bench_staging(device, reps=10)
+        line["staging"] = bench_staging(device, reps=10, layers=args.staging_layers)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:

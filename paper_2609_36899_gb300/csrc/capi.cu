@@ -70,17 +70,37 @@ EncodeTiledFn encode_tiled_fn()
     return fn;
 }
 
-// Tensor map over one layer's pages viewed as a 2-D bf16 matrix
-// [num_pages * Hkv * 16 rows][D columns]; box = 16 rows x 64 columns (128 B),
-// 128-byte swizzle so that ldmatrix reads of a page are bank-conflict free.
+// Tensor map over one layer's pages.  Preferred (D = 128): a 4-D view
+// {64 columns, 16 tokens, 2 column halves, page-heads} with strides
+// {256 B, 128 B, 16*D*2 B} and box {64, 16, 2, 1}, so one TMA op moves a whole
+// 4 KB (page, head) block and lands it as [half][token][64] -- two 16 x 128 B
+// panels, 128-byte swizzled so that ldmatrix reads are bank-conflict free.
+// Fallback (and D = 64): a 2-D view [rows = page-heads * 16][D] with a
+// 16 x 64 box, one op per 64-column panel.  *whole_block reports which.
 int encode_pages_map(CUtensorMap *map, const void *pages, int num_pages, int num_kv_heads,
-                     int head_dim)
+                     int head_dim, bool allow_whole, int *whole_block)
 {
     EncodeTiledFn fn = encode_tiled_fn();
     if (!fn)
         return CADKV_ERR_CUDA;
-    const cuuint64_t dims[2] = {(cuuint64_t)head_dim,
-                                (cuuint64_t)num_pages * num_kv_heads * kPageSize};
+    const cuuint64_t page_heads = (cuuint64_t)num_pages * num_kv_heads;
+    if (head_dim == 128 && allow_whole) {
+        const cuuint64_t dims[4] = {64, (cuuint64_t)kPageSize, 2, page_heads};
+        const cuuint64_t strides[3] = {(cuuint64_t)head_dim * 2, 128,
+                                       (cuuint64_t)kPageSize * head_dim * 2};
+        const cuuint32_t box[4] = {64, (cuuint32_t)kPageSize, 2, 1};
+        const cuuint32_t elem[4] = {1, 1, 1, 1};
+        CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(pages), dims,
+                        strides, box, elem, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r == CUDA_SUCCESS) {
+            *whole_block = 1;
+            return CADKV_OK;
+        }
+    }
+    *whole_block = 0;
+    const cuuint64_t dims[2] = {(cuuint64_t)head_dim, page_heads * kPageSize};
     const cuuint64_t strides[1] = {(cuuint64_t)head_dim * 2};
     const cuuint32_t box[2] = {64, (cuuint32_t)kPageSize};
     const cuuint32_t elem[2] = {1, 1};
@@ -197,9 +217,19 @@ int run_impl(const void *q, const void *k_pages, const void *v_pages,
     if (rc != CADKV_OK)
         return rc;
     CUtensorMap kmap, vmap;
-    if (encode_pages_map(&kmap, k_pages, s.num_pages, s.num_kv_heads, s.head_dim) != CADKV_OK ||
-        encode_pages_map(&vmap, v_pages, s.num_pages, s.num_kv_heads, s.head_dim) != CADKV_OK)
+    int k_whole = 0, v_whole = 0;
+    if (encode_pages_map(&kmap, k_pages, s.num_pages, s.num_kv_heads, s.head_dim, true,
+                         &k_whole) != CADKV_OK ||
+        encode_pages_map(&vmap, v_pages, s.num_pages, s.num_kv_heads, s.head_dim, true,
+                         &v_whole) != CADKV_OK)
         return CADKV_ERR_CUDA;
+    if (k_whole != v_whole) {  // both maps must use the same box shape
+        if (encode_pages_map(&kmap, k_pages, s.num_pages, s.num_kv_heads, s.head_dim, false,
+                             &k_whole) != CADKV_OK ||
+            encode_pages_map(&vmap, v_pages, s.num_pages, s.num_kv_heads, s.head_dim, false,
+                             &v_whole) != CADKV_OK)
+            return CADKV_ERR_CUDA;
+    }
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     AttnParams p{};
     p.q = static_cast<const __nv_bfloat16 *>(q);
@@ -218,6 +248,7 @@ int run_impl(const void *q, const void *k_pages, const void *v_pages,
     p.group = s.num_q_heads / s.num_kv_heads;
     p.max_pages = s.max_pages;
     p.num_pages = s.num_pages;
+    p.whole_page_box = k_whole && v_whole;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s.head_dim));
     return launch_attention(p, kmap, vmap, s.head_dim, sms, stream) == cudaSuccess ? CADKV_OK
                                                                                     : CADKV_ERR_CUDA;

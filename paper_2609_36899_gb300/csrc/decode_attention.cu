@@ -40,6 +40,7 @@ namespace cadkv {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
+constexpr int kIssueGroup = 8;  // pages the producer warp issues in parallel (<= stages)
 constexpr float kLn2 = 0.6931471805599453f;
 
 __host__ __device__ constexpr size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -202,6 +203,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 {
     using C = AttnConfig<D>;
     constexpr int S = C::kStages;
+    static_assert(kIssueGroup <= S, "a parallel issue group must not reuse a stage");
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(align_up(reinterpret_cast<size_t>(smem_raw), 1024));
     uint8_t *stages = smem + C::kStagesOff;
@@ -318,37 +320,62 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 ++sp;
 
                 const int *bt_row = p.block_table + (size_t)b * p.max_pages + j0;
+                // Block-table entries come 32 at a time, one chunk ahead of use.
+                int next_phys = lane < npg ? __ldg(bt_row + lane) : 0;
                 for (int c = 0; c < npg && ok; c += 32) {
-                    int phys = 0;
+                    int phys = next_phys;
+                    if (c + 32 + lane < npg)
+                        next_phys = __ldg(bt_row + c + 32 + lane);
                     if (c + lane < npg) {
-                        phys = bt_row[c + lane];
                         if (phys < 0 || phys >= p.num_pages) {
                             record_status(&p.hdr->status, CADKV_ERR_OOB);
                             phys = 0;
                         }
                     }
                     const int cnt = min(32, npg - c);
-                    for (int i = 0; i < cnt; ++i) {
-                        const int ph = __shfl_sync(kFull, phys, i);
-                        const uint32_t st = kp % S;
-                        if (kp >= (uint32_t)S) {
-                            ok = mbar_wait(&empty_bar[st], ((kp / S) + 1) & 1, abort_flag);
-                            ok = __all_sync(kFull, ok);
-                            if (!ok)
-                                break;
-                        }
-                        if (lane == 0) {
-                            uint8_t *kdst = stages + (size_t)st * C::kStageBytes;
-                            uint8_t *vdst = kdst + C::kKBytes;
-                            const int y = (ph * Hkv + kvh) * kPageSize;
-                            mbar_arrive_expect_tx(&full_bar[st], C::kStageBytes);
+                    // Issue kIssueGroup pages at once, one lane per page: each lane
+                    // waits for its own stage to be released and starts its own
+                    // copies, so the mbarrier and TMA-issue latencies of a group
+                    // overlap instead of adding up page after page.
+                    for (int i0 = 0; i0 < cnt; i0 += kIssueGroup) {
+                        const int gcnt = min(kIssueGroup, cnt - i0);
+                        const int ph = __shfl_sync(kFull, phys, (i0 + lane) & 31);
+                        const uint32_t kl = kp + lane;
+                        const uint32_t st = kl % S;
+                        bool lok = true;
+                        if (lane < gcnt) {
+                            if (kl >= (uint32_t)S)
+                                lok = mbar_wait(&empty_bar[st], ((kl / S) + 1) & 1, abort_flag);
+                            if (lok) {
+                                uint8_t *kdst = stages + (size_t)st * C::kStageBytes;
+                                uint8_t *vdst = kdst + C::kKBytes;
+                                const int ph_head = ph * Hkv + kvh;
+                                mbar_arrive_expect_tx(&full_bar[st], C::kStageBytes);
+                                if (C::kBoxes > 1 && p.whole_page_box) {
+                                    // one 4 KB op per block: box {64 cols, 16 tokens, 2 halves}
+                                    tma_load_4d(kdst, &kmap, 0, 0, 0, ph_head, &full_bar[st], policy);
+                                    tma_load_4d(vdst, &vmap, 0, 0, 0, ph_head, &full_bar[st], policy);
+                                } else {
 #pragma unroll
-                            for (int bx = 0; bx < C::kBoxes; ++bx) {
-                                tma_load_2d(kdst + bx * C::kBoxBytes, &kmap, bx * 64, y, &full_bar[st], policy);
-                                tma_load_2d(vdst + bx * C::kBoxBytes, &vmap, bx * 64, y, &full_bar[st], policy);
+                                    for (int bx = 0; bx < C::kBoxes; ++bx) {
+                                        tma_load_2d(kdst + bx * C::kBoxBytes, &kmap, bx * 64,
+                                                    ph_head * kPageSize, &full_bar[st], policy);
+                                        tma_load_2d(vdst + bx * C::kBoxBytes, &vmap, bx * 64,
+                                                    ph_head * kPageSize, &full_bar[st], policy);
+                                    }
+                                }
                             }
                         }
-                        ++kp;
+                        ok = __all_sync(kFull, lok);
+                        if (!ok) {
+                            // copies this group did start must land before we leave
+                            if (lane < gcnt && lok) {
+                                volatile int never = 0;
+                                mbar_wait(&full_bar[st], (kl / S) & 1, &never);
+                            }
+                            break;
+                        }
+                        kp += gcnt;
                     }
                 }
                 if (!ok)
@@ -367,6 +394,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 desc[r].num_pages = -1;
                 mbar_arrive(&seg_full[r]);
             }
+            if (ok)
+                ++sp;  // the sentinel occupies a ring slot like any segment
         }
         if (!ok && lane == 0) {
             *abort_flag = 1;
@@ -426,8 +455,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
 
         const int npg = d.num_pages;
-        const int i0 = (int)((warp + kNumConsumerWarps - (int)(k % kNumConsumerWarps)) % kNumConsumerWarps);
-        for (int i = i0; i < npg; i += kNumConsumerWarps) {
+        // Page i of a segment always goes to warp i % 4, whatever the CTA did
+        // before, so the summation order (and the result) is deterministic.
+        for (int i = warp; i < npg; i += kNumConsumerWarps) {
             const uint32_t kk_idx = k + i;
             const uint32_t st = kk_idx % S;
             ok = __all_sync(kFull, mbar_wait(&full_bar[st], (kk_idx / S) & 1, abort_flag));

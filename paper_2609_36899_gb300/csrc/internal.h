@@ -7,7 +7,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
-#include "../../include/cadkv.h"
+#include "cadkv.h"
 
 namespace cadkv {
 
@@ -68,7 +68,8 @@ struct AttnParams {
     float *part_lse;
     float *part_o;
     int batch, num_q_heads, num_kv_heads, group, max_pages, num_pages;
-    float scale_log2;  // log2(e) / sqrt(D)
+    int whole_page_box;  // 1: the tensor maps copy a whole (page, head) block per TMA op
+    float scale_log2;    // log2(e) / sqrt(D)
 };
 
 cudaError_t launch_plan(const PlanParams &p, cudaStream_t stream);
