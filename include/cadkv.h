@@ -224,6 +224,48 @@ int kv_prefix_load(const cadkv_pool *pool, const int32_t *block_table, int max_p
 /* As decode_attention_status, for a staging/load workspace. */
 int kv_prefix_stage_status(const void *workspace, cadkv_stream_t stream);
 
+/* ------------------------------------------------------------------------ */
+/* Decode attention without caller-provided scratch                          */
+/* ------------------------------------------------------------------------ */
+
+/* Size of the scratch array decode_attention_noalloc uses (32 MiB). */
+#define CADKV_NOALLOC_SCRATCH_BYTES (32u << 20)
+
+/*
+ * decode_attention for callers that cannot allocate device memory when they
+ * call it.  (The paper has no counterpart; this is a library convenience.)
+ * Examples: a serving engine that reserved nearly all HBM for its KV cache at
+ * start-up, so a cudaMalloc at call time would fail or fragment that pool; or
+ * a plugin that has no handle on its host framework's allocator and must not
+ * call cudaMalloc/cudaFree itself (cudaFree also synchronises the device).
+ *
+ * Arguments and results are those of decode_attention without the workspace:
+ * the caller still passes every input and output.  The scratch space the
+ * computation needs (page prefix sums, arrival counters, split partials) lives
+ * in one file-scope device array of CADKV_NOALLOC_SCRATCH_BYTES, which every
+ * GPU that loads the library holds until the process exits.  Nothing is
+ * allocated: no cudaMalloc, no cudaFree, no allocating library routine.
+ *
+ * - The first call on a device looks up that device's address of the array
+ *   (cudaGetSymbolAddress, with the device current) and caches it; make that
+ *   first call before any stream capture on the device.
+ * - A problem whose scratch would exceed CADKV_NOALLOC_SCRATCH_BYTES is
+ *   rejected with CADKV_ERR_WORKSPACE before anything is launched (the
+ *   requirement is decode_attention_workspace_size() of the same sizes).
+ * - Every call on a device shares the one array, and the array keeps the last
+ *   call's contents; each call's planner clears what must start at zero
+ *   (status word, work counter, arrival counters) itself.  Calls whose
+ *   kernels may overlap on the GPU (different streams without ordering) race
+ *   on the array and give wrong results: order them on one stream.
+ * - The device status word of the last call is not exposed by this entry
+ *   point; use decode_attention with a workspace when it is needed.
+ */
+int decode_attention_noalloc(const void *q, const void *k_pages, const void *v_pages,
+                             const int32_t *block_table, const int32_t *context_lens,
+                             void *out, float *lse, int batch, int num_q_heads,
+                             int num_kv_heads, int head_dim, int page_size, int num_pages,
+                             int max_pages, cadkv_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -57,6 +57,8 @@ _SIGNATURES = {
     "decode_attention_run": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I,
                                   _P, _SZ, _P]),
     "decode_attention_status": (_I, [_P, _P]),
+    "decode_attention_noalloc": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I,
+                                      _P]),
     "kv_prefix_stage_workspace_size": (_SZ, [_I]),
     "kv_prefix_stage": (_I, [_P, _P, _I, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
     "kv_prefix_load": (_I, [_P, _P, _I, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
@@ -216,6 +218,25 @@ def decode_attention_status(workspace, stream=None) -> int:
     """Synchronise the stream and return the device status word (0 = ok)."""
     return int(library().decode_attention_status(_ptr(workspace),
                                                  _stream(stream, workspace.device)))
+
+
+def decode_attention_noalloc(q, k_pages, v_pages, block_table, context_lens, out=None,
+                             lse=None, want_lse: bool = True, stream=None):
+    """decode_attention using the library's built-in scratch array instead of
+    a workspace, for callers that cannot allocate device memory at call time
+    (outputs are still allocated here when not given)."""
+    batch, hq, hkv, d, page, num_pages, max_pages = _decode_args(
+        q, k_pages, v_pages, block_table, context_lens)
+    if out is None:
+        out = torch.empty_like(q)
+    if lse is None and want_lse:
+        lse = torch.empty((batch, hq), dtype=torch.float32, device=q.device)
+    rc = library().decode_attention_noalloc(
+        _ptr(q), _ptr(k_pages), _ptr(v_pages), _ptr(block_table), _ptr(context_lens),
+        _ptr(out), _ptr(lse), batch, hq, hkv, d, page, num_pages, max_pages,
+        _stream(stream, q.device))
+    _check("decode_attention_noalloc", rc)
+    return out, lse
 
 
 # ------------------------------------------------------------------ pool + staging

@@ -522,6 +522,75 @@ int decode_attention_status(const void *workspace, cadkv_stream_t stream)
     return read_status(workspace, reinterpret_cast<cudaStream_t>(stream));
 }
 
+}  // extern "C"
+
+// Scratch of decode_attention_noalloc: one array per device, never allocated
+// at call time.  Host code may only use its device address, obtained with
+// cudaGetSymbolAddress while that device is current (the name itself is a
+// host-side stand-in).
+static __device__ __align__(256) unsigned char g_noalloc_scratch[CADKV_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+
+// Device address of g_noalloc_scratch on the current device, looked up once
+// per device and cached.
+int noalloc_scratch(void **ptr)
+{
+    static std::mutex mu;
+    static void *cache[64] = {nullptr};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64)
+        return CADKV_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!cache[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p)
+            return CADKV_ERR_CUDA;
+        cache[dev] = p;
+    }
+    *ptr = cache[dev];
+    return CADKV_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int decode_attention_noalloc(const void *q, const void *k_pages, const void *v_pages,
+                             const int32_t *block_table, const int32_t *context_lens, void *out,
+                             float *lse, int batch, int num_q_heads, int num_kv_heads,
+                             int head_dim, int page_size, int num_pages, int max_pages,
+                             cadkv_stream_t stream)
+{
+    const DecodeShape s{batch, num_q_heads, num_kv_heads, head_dim, page_size, num_pages, max_pages};
+    int rc = check_decode_shape(s);
+    if (rc != CADKV_OK)
+        return rc;
+    if (batch == 0)
+        return CADKV_OK;
+    rc = check_run_args(q, k_pages, v_pages, block_table, context_lens, out, lse, s);
+    if (rc != CADKV_OK)
+        return rc;
+    const int sms = device_sms();
+    if (sms < 0)
+        return sms;
+    const size_t need = decode_workspace_layout(batch, num_kv_heads, num_q_heads / num_kv_heads,
+                                                head_dim, sms)
+                            .total;
+    if (need > (size_t)CADKV_NOALLOC_SCRATCH_BYTES)
+        return CADKV_ERR_WORKSPACE;
+    void *scratch = nullptr;
+    rc = noalloc_scratch(&scratch);
+    if (rc != CADKV_OK)
+        return rc;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    rc = plan_impl(context_lens, out, lse, s, 0, scratch, CADKV_NOALLOC_SCRATCH_BYTES, st);
+    if (rc != CADKV_OK)
+        return rc;
+    return run_impl(q, k_pages, v_pages, block_table, context_lens, out, lse, s, scratch,
+                    CADKV_NOALLOC_SCRATCH_BYTES, st);
+}
+
 size_t kv_prefix_stage_workspace_size(int batch)
 {
     if (batch < 0)
