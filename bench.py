@@ -48,7 +48,7 @@ NOMINAL_HBM_GBS = 8000.0
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
 PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "decode_attention_kernel_paced_b256.md")
-STAGE_PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "prefix_stage_copy_64traj.md")
+STAGE_PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "stage_copy_kernel_staging_8traj_1layer.md")
 KERNEL_SOURCE = os.path.join(ROOT, "paper_2609_36899_gb300", "csrc", "decode_attention.cu")
 STAGE_SOURCE = os.path.join(ROOT, "paper_2609_36899_gb300", "csrc", "prefix_stage.cu")
 
