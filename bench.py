@@ -40,8 +40,8 @@ sys.path.insert(0, ROOT)
 import paper_2609_36899_gb300 as cadkv  # noqa: E402
 from paper_2609_36899_gb300 import build as pkg_build  # noqa: E402
 from paper_2609_36899_gb300.workloads import (DECODE_WORKLOADS, STAGING, bf16_bits,  # noqa: E402
-                                              fill_layer_pool, make_decode_batch,
-                                              make_staging_job)
+                                              fill_layer_pool, landscape_workload,
+                                              make_decode_batch, make_staging_job)
 
 METRIC = "decode-attention achieved HBM GB/s (% of 8 TB/s) and decode steps/s per batch"
 NOMINAL_HBM_GBS = 8000.0
@@ -332,6 +332,15 @@ def bench_staging(device, reps, layers=2, batch=None):
     torch.cuda.synchronize()
     status = cadkv.kv_prefix_stage_status(ws)
     ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in ev)
+    # the inverse direction: load the staged rows back into the same pages
+    # (the values written equal the values already there)
+    for e0, e1 in ev:
+        e0.record(stream)
+        cadkv.kv_prefix_load(pool, bt, cl, 0, layers, dst, workspace=ws, stream=stream)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    load_status = cadkv.kv_prefix_stage_status(ws)
+    load_ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in ev)
     moved = 2 * size * 2  # read + write, bytes
     # bit-exact spot check of one trajectory's staged rows against the pool
     b = int(np.argmax(lens))
@@ -352,6 +361,9 @@ def bench_staging(device, reps, layers=2, batch=None):
            "bytes_per_call": moved, "launches_per_call": 2, "status": status,
            "bit_exact_spot_check": ok,
            "full_job_ms_estimate": round(ms * 48 / layers, 1),
+           "load": {"gbps_read_plus_write": round(moved / (load_ms * 1e-3) / 1e9, 1),
+                    "ms_per_call": round(load_ms, 3), "status": load_status,
+                    "frac_of_copy_peak": round(moved / (load_ms * 1e-3) / 1e9 / hbm_peak()[0], 4)},
            "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": peak,
                         "unit": "GB/s", "frac": round(gbs / peak, 4),
                         "peak_kind": kind,
@@ -359,6 +371,49 @@ def bench_staging(device, reps, layers=2, batch=None):
     del dst, k_layers, v_layers, pool
     torch.cuda.empty_cache()
     return res
+
+
+def read_probe(buf, reps=10):
+    """Pure-read bandwidth (GB/s) of ``buf`` with the library's read probe."""
+    sink = torch.zeros(1, dtype=torch.int64, device=buf.device)
+    stream = torch.cuda.current_stream(buf.device)
+    for _ in range(3):
+        cadkv.cadkv_hbm_read_probe(buf, sink, stream=stream)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        cadkv.cadkv_hbm_read_probe(buf, sink, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return buf.numel() * buf.element_size() * reps / (e0.elapsed_time(e1) * 1e-3) / 1e9
+
+
+def bench_landscape(device, steps, warmup, batches=(8, 32, 128, 512),
+                    means=(1024, 4096, 16384, 65536), max_tokens=8 << 20):
+    """Decode GB/s and steps/s over (B, mean context), 32/8 heads, D = 128."""
+    cells = []
+    for b in batches:
+        for c in means:
+            if b * c > max_tokens:
+                continue
+            w = landscape_workload(b, c)
+            batch = make_decode_batch(w, device=device)
+            tensors = _tensors(batch, device)
+            stream = torch.cuda.current_stream(device)
+            ev = time_decode(tensors, steps, warmup, stream)
+            run_decode_loop(tensors, ev, stream)
+            torch.cuda.synchronize()
+            step_ms = ev[0][0].elapsed_time(ev[-1][2]) / steps
+            nbytes = decode_bytes(batch.context_lens, w.num_q_heads, w.num_kv_heads, w.head_dim)
+            cells.append({"batch": b, "mean_context": c,
+                          "gbps": round(nbytes / (step_ms * 1e-3) / 1e9, 1),
+                          "ms_per_step": round(step_ms, 4),
+                          "steps_per_s": round(1e3 / step_ms, 1),
+                          "tokens_per_s_per_layer": round(b * 1e3 / step_ms, 1),
+                          "status": cadkv.decode_attention_status(tensors[7])})
+            del batch, tensors
+            torch.cuda.empty_cache()
+    return cells
 
 
 def bench_config(name, device, steps, warmup):
@@ -405,7 +460,7 @@ def main():
     ap.add_argument("--steps", type=int, default=400)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=sorted(DECODE_WORKLOADS) + ["staging"],
+    ap.add_argument("--workload", choices=sorted(DECODE_WORKLOADS) + ["staging", "landscape"],
                     default="mixed",
                     help="decode workload of the headline line, or 'staging' to time "
                          "only prefix staging")
@@ -433,6 +488,13 @@ def main():
                             batch=args.staging_batch)
         if rank == 0:
             print(json.dumps(res), flush=True)
+        return
+    if args.workload == "landscape":
+        cells = bench_landscape(device, args.steps, args.warmup)
+        if rank == 0:
+            print(json.dumps({"workload": "decode-throughput landscape over (B, mean context), "
+                                          "32/8 heads, D=128, lengths U[C/2, 3C/2]",
+                              "unit": "GB/s", "cells": cells}), flush=True)
         return
     w = DECODE_WORKLOADS[args.workload]
     batch = make_decode_batch(w, device=device, seed=w.seed + rank)
@@ -465,6 +527,7 @@ def main():
 
     peak, kind = hbm_peak()
     achieved = nbytes / (kern_ms * 1e-3) / 1e9
+    read_gbps = read_probe(batch.k_pages)
     line = {
         "metric": METRIC,
         "value": round(value, 1),
@@ -498,6 +561,8 @@ def main():
                      "unit": "GB/s", "frac": round(achieved / peak, 4),
                      "peak_kind": kind, "kernel": "decode_attention_kernel<128>",
                      "kernel_ms": round(kern_ms, 4), "planner_ms": round(plan_ms, 4),
+                     "read_probe_gbps": round(read_gbps, 1),
+                     "frac_of_read_probe": round(achieved / read_gbps, 4),
                      "traffic": profiled_traffic(PROFILE_SUMMARY, KERNEL_SOURCE)},
         "clocks": clocks,
         "device_status": status,

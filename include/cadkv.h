@@ -224,6 +224,16 @@ int kv_prefix_load(const cadkv_pool *pool, const int32_t *block_table, int max_p
 /* As decode_attention_status, for a staging/load workspace. */
 int kv_prefix_stage_status(const void *workspace, cadkv_stream_t stream);
 
+/*
+ * Measuring aid (no counterpart in the paper): read `bytes` (a multiple of 16)
+ * of device memory `buf` with 16-byte streaming loads and XOR them into the
+ * device word *sink (8-byte aligned; the caller zeroes it).  The only DRAM
+ * traffic is the read, so bytes / time is the read-bandwidth ceiling that the
+ * read-dominated decode-attention stream is compared with.
+ */
+int cadkv_hbm_read_probe(const void *buf, size_t bytes, unsigned long long *sink,
+                         cadkv_stream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* Decode attention without caller-provided scratch                          */
 /* ------------------------------------------------------------------------ */

@@ -63,6 +63,7 @@ _SIGNATURES = {
     "kv_prefix_stage": (_I, [_P, _P, _I, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
     "kv_prefix_load": (_I, [_P, _P, _I, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
     "kv_prefix_stage_status": (_I, [_P, _P]),
+    "cadkv_hbm_read_probe": (_I, [_P, _SZ, _P, _P]),
 }
 
 _lib = None
@@ -336,6 +337,17 @@ def kv_prefix_load(pool: KVPool, block_table, context_lens, layer_begin: int,
     return _stage_common(library().kv_prefix_load, "kv_prefix_load", pool, block_table,
                          context_lens, layer_begin, layer_end, src, src_offsets, workspace,
                          stream)
+
+
+def cadkv_hbm_read_probe(buf, sink, stream=None):
+    """Read all of ``buf`` (a CUDA tensor, size a multiple of 16 bytes) and XOR
+    it into ``sink`` (an int64 CUDA tensor of one element, zeroed by the caller)."""
+    if not buf.is_cuda or not buf.is_contiguous():
+        raise ValueError("buf must be a contiguous CUDA tensor")
+    _need(sink, "sink", torch.int64, 1, buf.device)
+    rc = library().cadkv_hbm_read_probe(_ptr(buf), buf.numel() * buf.element_size(),
+                                        _ptr(sink), _stream(stream, buf.device))
+    _check("cadkv_hbm_read_probe", rc)
 
 
 def kv_prefix_stage_status(workspace, stream=None) -> int:

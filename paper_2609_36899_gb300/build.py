@@ -19,7 +19,7 @@ CSRC = PKG / "csrc"
 INCLUDE = PKG.parent / "include"
 BUILD_DIR = PKG / "_build"
 LIBRARY = PKG / "libcadkv.so"
-SOURCES = ["capi.cu", "decode_attention.cu", "prefix_stage.cu"]
+SOURCES = ["capi.cu", "decode_attention.cu", "prefix_stage.cu", "hbm_probe.cu"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC",

@@ -623,4 +623,20 @@ int kv_prefix_stage_status(const void *workspace, cadkv_stream_t stream)
     return read_status(workspace, reinterpret_cast<cudaStream_t>(stream));
 }
 
+int cadkv_hbm_read_probe(const void *buf, size_t bytes, unsigned long long *sink,
+                         cadkv_stream_t stream)
+{
+    if (!buf || !sink || !aligned(buf, 16) || !aligned(sink, 8) || bytes % 16 != 0)
+        return CADKV_ERR_INVALID;
+    if (bytes == 0)
+        return CADKV_OK;
+    const int sms = device_sms();
+    if (sms < 0)
+        return sms;
+    return launch_hbm_read(buf, bytes, sink, sms, reinterpret_cast<cudaStream_t>(stream)) ==
+                   cudaSuccess
+               ? CADKV_OK
+               : CADKV_ERR_CUDA;
+}
+
 }  // extern "C"

@@ -103,4 +103,7 @@ StageWorkspaceLayout stage_workspace_layout(int batch);
 
 cudaError_t launch_stage(const StageParams &p, int num_sms, cudaStream_t stream);
 
+cudaError_t launch_hbm_read(const void *src, size_t bytes, unsigned long long *sink,
+                            int num_sms, cudaStream_t stream);
+
 }  // namespace cadkv

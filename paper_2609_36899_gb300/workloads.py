@@ -79,6 +79,15 @@ DECODE_WORKLOADS = {"tiny": TINY, "paced": PACED, "long_tail": LONG_TAIL,
                     "mixed": MIXED}
 
 
+def landscape_workload(batch: int, mean_len: int, seed: int = 20266) -> DecodeWorkload:
+    """One cell of the decode-throughput landscape over (B, mean context C):
+    lengths uniform in [C/2, 3C/2], 32 query / 8 KV heads, head_dim 128 (the
+    head geometry of the paper's Qwen3-8B runs)."""
+    lo, hi = mean_len // 2, (3 * mean_len) // 2
+    return DecodeWorkload(f"landscape B={batch} C={mean_len}", batch, 32, 8, 128, "uniform",
+                          (lo, hi), hi, seed + batch * 1000003 + mean_len)
+
+
 def draw_lengths(kind: str, args: tuple, batch: int,
                  rng: np.random.Generator) -> np.ndarray:
     """Context lengths n_b (int32)."""

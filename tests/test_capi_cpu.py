@@ -95,3 +95,12 @@ def test_stage_rejects_null_pool(lib):
     P = ctypes.c_void_p
     assert lib.kv_prefix_stage(None, P(1 << 12), 4, P(1 << 12), 2, 0, 1, P(1 << 12), None,
                                P(1 << 12), 1 << 20, None) == STATUS["CADKV_ERR_INVALID"]
+
+
+def test_read_probe_rejects_on_host(lib):
+    P = ctypes.c_void_p
+    assert lib.cadkv_hbm_read_probe(None, 16, P(1 << 12), None) == STATUS["CADKV_ERR_INVALID"]
+    assert lib.cadkv_hbm_read_probe(P(1 << 12), 15, P(1 << 12), None) == STATUS["CADKV_ERR_INVALID"]
+    assert lib.cadkv_hbm_read_probe(P((1 << 12) + 4), 16, P(1 << 12), None) == \
+        STATUS["CADKV_ERR_INVALID"]
+    assert lib.cadkv_hbm_read_probe(P(1 << 12), 0, P(1 << 12), None) == 0

@@ -231,3 +231,33 @@ def test_workspace_too_small_is_rejected():
     with pytest.raises(cadkv.CadkvError) as e:
         cadkv.decode_attention(q, k, v, bt, cl, workspace=ws)
     assert e.value.status == STATUS["CADKV_ERR_WORKSPACE"]
+
+
+@pytest.mark.parametrize("b,c", [(32, 16384), (8, 65536), (512, 1024)])
+def test_landscape_cells_sampled(b, c):
+    """Cells of the (B, mean context) landscape sweep, full size, sampled rows."""
+    from paper_2609_36899_gb300.workloads import landscape_workload
+    w = landscape_workload(b, c)
+    batch = make_decode_batch(w, device="cuda")
+    tensors = (batch.q, batch.k_pages, batch.v_pages,
+               torch.from_numpy(batch.block_table).cuda(),
+               torch.from_numpy(batch.context_lens).cuda())
+    out, lse = gpu_decode(batch, tensors=tensors)
+    lens = batch.context_lens
+    sample = sorted({int(np.argmax(lens)), int(np.argmin(lens)), len(lens) // 2})
+    ref, ref_lse = sampled_oracle(batch, sample)
+    idx = torch.tensor(sample, device="cuda")
+    assert_close(out[idx], lse[idx], ref, ref_lse, w.name)
+
+
+def test_hbm_read_probe_reads_every_word():
+    g = torch.Generator().manual_seed(1)
+    host = torch.randint(-2**31, 2**31 - 1, (1 << 20,), generator=g, dtype=torch.int64)
+    host = host.to(torch.int32)
+    buf = host.cuda()
+    sink = torch.zeros(1, dtype=torch.int64, device="cuda")
+    cadkv.cadkv_hbm_read_probe(buf, sink)
+    torch.cuda.synchronize()
+    expect = int(np.bitwise_xor.reduce(host.numpy().view(np.uint32)))
+    assert int(sink.item()) & 0xFFFFFFFF == expect
+    assert int(sink.item()) >> 32 == 0
