@@ -20,6 +20,8 @@ Definitions (written out in ``oracle.c``):
   (Sec. 4.4, phase 1).
 * ``prefix_load`` -- its inverse, the destination-side materialisation of a
   staged prefix into a paged pool (Sec. 4.4, phase 3).
+* ``kv_append`` -- the write of each trajectory's new-token key and value
+  into its paged cache that precedes attention in every decode step.
 
 Every function is pinned by the CPU tests in ``tests/test_oracle_*.py``.
 """
@@ -100,6 +102,9 @@ class Oracle:
         f.restype = ctypes.c_int
         f.argtypes = [_P, _P, _I64, _I64, _I64, _I64, _I64, _P, _I64, _P, _I64,
                       _I64, _I64, _P, _P]
+        f = self.lib.oracle_kv_append
+        f.restype = ctypes.c_int
+        f.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64, _I64]
         self.lib.oracle_max_threads.restype = ctypes.c_int
 
     def max_threads(self) -> int:
@@ -194,6 +199,24 @@ class Oracle:
         self._check(rc)
         return k_pool, v_pool
 
+    def kv_append(self, k_pages, v_pages, k_new, v_new, block_table, context_lens):
+        """Write the new token's K/V rows (uint16 [B, Hkv, D]) into ``k_pages`` /
+        ``v_pages`` (uint16 [num_pages, Hkv, P, D], C-contiguous) in place."""
+        for name, a in (("k_pages", k_pages), ("v_pages", v_pages)):
+            if a.dtype != np.uint16 or not a.flags.c_contiguous:
+                raise TypeError(f"{name} must be a C-contiguous uint16 array")
+        k_new, v_new = _u16(k_new), _u16(v_new)
+        block_table, context_lens = _i32(block_table), _i32(context_lens)
+        num_pages, hkv, page, d = k_pages.shape
+        if k_new.shape != (context_lens.shape[0], hkv, d) or v_new.shape != k_new.shape:
+            raise ValueError("k_new / v_new must be [B, Hkv, D]")
+        rc = self.lib.oracle_kv_append(
+            _ptr(k_pages), _ptr(v_pages), _ptr(k_new), _ptr(v_new), _ptr(block_table),
+            _ptr(context_lens), context_lens.shape[0], hkv, d, page, num_pages,
+            block_table.shape[1])
+        self._check(rc)
+        return k_pages, v_pages
+
 
 _DEFAULT: Oracle | None = None
 
@@ -215,3 +238,7 @@ def prefix_stage(*args, **kwargs):
 
 def prefix_load(*args, **kwargs):
     return default().prefix_load(*args, **kwargs)
+
+
+def kv_append(*args, **kwargs):
+    return default().kv_append(*args, **kwargs)

@@ -47,6 +47,13 @@
  *    following a destination block table.  Token slots of the last page past
  *    n_b are left untouched.
  *
+ * 4. oracle_kv_append: the step that precedes attention in every decode step
+ *    (Sec. 2.3: each step appends the new token's key and value to the
+ *    trajectory's KV cache): for every trajectory with n_b >= 1 and KV head h,
+ *    the new token's rows k_new[b][h][:] and v_new[b][h][:] are written to
+ *    token position n_b - 1, i.e. page block_table[b][(n_b - 1) / P], slot
+ *    (n_b - 1) % P.  Trajectories with n_b = 0 append nothing.
+ *
  * Pool layout: per layer, K and V are each [num_pages][Hkv][P][D] bf16
  * (head-major inside a page); layers are stacked with stride
  * num_pages * Hkv * P * D elements.
@@ -294,6 +301,41 @@ int oracle_prefix_load(uint16_t *k_pool, uint16_t *v_pool, int64_t num_layers,
                     }
                 }
             }
+    }
+    return 0;
+}
+
+/*
+ * k_new, v_new: [B][Hkv][D] bf16 bits; k_pages, v_pages: [num_pages][Hkv][P][D]
+ * (one layer), updated in place.
+ */
+int oracle_kv_append(uint16_t *k_pages, uint16_t *v_pages, const uint16_t *k_new,
+                     const uint16_t *v_new, const int32_t *block_table,
+                     const int32_t *context_lens, int64_t batch, int64_t num_kv_heads,
+                     int64_t head_dim, int64_t page_size, int64_t num_pages,
+                     int64_t max_pages)
+{
+    if (!k_pages || !v_pages || !k_new || !v_new || !block_table || !context_lens)
+        return -1;
+    int rc = check_lengths(block_table, context_lens, batch, page_size, num_pages,
+                           max_pages);
+    if (rc != 0)
+        return rc;
+    for (int64_t b = 0; b < batch; ++b) {
+        const int64_t n = context_lens[b];
+        if (n == 0)
+            continue;
+        const int64_t t = n - 1;
+        const int64_t phys = block_table[b * max_pages + t / page_size];
+        const int64_t slot = t % page_size;
+        for (int64_t h = 0; h < num_kv_heads; ++h) {
+            const int64_t dst = ((phys * num_kv_heads + h) * page_size + slot) * head_dim;
+            const int64_t src = (b * num_kv_heads + h) * head_dim;
+            for (int64_t d = 0; d < head_dim; ++d) {
+                k_pages[dst + d] = k_new[src + d];
+                v_pages[dst + d] = v_new[src + d];
+            }
+        }
     }
     return 0;
 }

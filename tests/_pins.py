@@ -398,3 +398,67 @@ def pin_stage_round_trip(orc):
 
 
 STAGE_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_stage_")]
+
+
+# --------------------------------------------------------------------------
+# KV append
+# --------------------------------------------------------------------------
+
+def pin_append_then_attend_matches_scipy(orc):
+    """Appending the new token's K/V and attending equals scipy attention over
+    the logical rows with the new token as the last row."""
+    lens_old = [16, 0, 40, 5]
+    hq, hkv, d = 8, 2, 64
+    rng = _rng(50)
+    ks = [to_bf16_bits(rng.normal(size=(n + 1, hkv, d))) for n in lens_old]
+    vs = [to_bf16_bits(rng.normal(size=(n + 1, hkv, d))) for n in lens_old]
+    q = to_bf16_bits(rng.normal(size=(len(lens_old), hq, d)))
+    # pool holds the old rows plus junk in the slot the new token goes to
+    junk_k = [np.concatenate([k[:-1], np.full((1, hkv, d), NAN_BF16, np.uint16)]) for k in ks]
+    junk_v = [np.concatenate([v[:-1], np.full((1, hkv, d), NAN_BF16, np.uint16)]) for v in vs]
+    used = sum(-(-(n + 1) // 16) for n in lens_old)
+    perm = rng.permutation(used + 2)
+    kp, table, cl = paged(junk_k, 16, perm, used + 2, fill=NAN_BF16)
+    vp, _, _ = paged(junk_v, 16, perm, used + 2, fill=NAN_BF16)
+    k_new = np.stack([k[-1] for k in ks])
+    v_new = np.stack([v[-1] for v in vs])
+    orc.kv_append(kp, vp, k_new, v_new, table, cl)
+    out, lse = orc.decode_attention(q, kp, vp, table, cl)
+    ref, ref_lse = _scipy_reference(q, ks, vs, hq, hkv)
+    np.testing.assert_allclose(out, ref, rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(lse, ref_lse, rtol=1e-12, atol=1e-12)
+
+
+def pin_append_writes_only_the_new_slot(orc):
+    """Append changes exactly the (page, head, slot) of token n_b - 1 of every
+    non-empty trajectory, to the new bits, and nothing else."""
+    lens = [1, 16, 17, 0, 33]
+    hkv, d = 3, 8
+    rng = _rng(51)
+    used = sum(-(-n // 16) for n in lens)
+    table = np.full((len(lens), 3), -1, dtype=np.int32)
+    perm = rng.permutation(used + 2)
+    pos = 0
+    for b, n in enumerate(lens):
+        p = -(-n // 16)
+        table[b, :p] = perm[pos:pos + p]
+        pos += p
+    kp = rng.integers(0, 1 << 16, size=(used + 2, hkv, 16, d), dtype=np.uint16)
+    vp = rng.integers(0, 1 << 16, size=(used + 2, hkv, 16, d), dtype=np.uint16)
+    k0, v0 = kp.copy(), vp.copy()
+    k_new = rng.integers(0, 1 << 16, size=(len(lens), hkv, d), dtype=np.uint16)
+    v_new = rng.integers(0, 1 << 16, size=(len(lens), hkv, d), dtype=np.uint16)
+    orc.kv_append(kp, vp, k_new, v_new, table, np.array(lens, dtype=np.int32))
+    changed = np.zeros(kp.shape[:3], dtype=bool)
+    for b, n in enumerate(lens):
+        if n == 0:
+            continue
+        ph, sl = table[b, (n - 1) // 16], (n - 1) % 16
+        np.testing.assert_array_equal(kp[ph, :, sl], k_new[b])
+        np.testing.assert_array_equal(vp[ph, :, sl], v_new[b])
+        changed[ph, :, sl] = True
+    np.testing.assert_array_equal(kp[~changed], k0[~changed])
+    np.testing.assert_array_equal(vp[~changed], v0[~changed])
+
+
+APPEND_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_append_")]

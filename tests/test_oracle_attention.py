@@ -38,3 +38,11 @@ def test_attention_thread_count_does_not_change_result(orc):
     b = orc.decode_attention(q, kp, vp, table, cl, num_threads=4)
     np.testing.assert_array_equal(a[0], b[0])
     np.testing.assert_array_equal(a[1], b[1])
+
+
+from _pins import APPEND_PINS  # noqa: E402
+
+
+@pytest.mark.parametrize("pin", APPEND_PINS, ids=lambda f: f.__name__)
+def test_append_pin(orc, pin):
+    pin(orc)

@@ -15,11 +15,12 @@ import re
 import pytest
 
 import oracle
-from _pins import ATTENTION_PINS, STAGE_PINS
+from _pins import APPEND_PINS, ATTENTION_PINS, STAGE_PINS
 
 ATT = "oracle_decode_attention"
 STAGE = "oracle_prefix_stage"
 LOAD = "oracle_prefix_load"
+APPEND = "oracle_kv_append"
 
 MUTANTS = [
     # (id, function, old, new, count) -- count 0 replaces every occurrence
@@ -58,6 +59,11 @@ MUTANTS = [
     ("load_tokens_reversed", LOAD,
      "memcpy(d, row + t * head_dim", "memcpy(d, row + (n - 1 - t) * head_dim", 1),
     ("load_k_v_swapped", LOAD, "(kv == 0 ? k_pool : v_pool)", "(kv == 1 ? k_pool : v_pool)", 1),
+    ("append_to_first_token", APPEND, "const int64_t t = n - 1;", "const int64_t t = 0;", 1),
+    ("append_head_reversed", APPEND,
+     "const int64_t src = (b * num_kv_heads + h) * head_dim;",
+     "const int64_t src = (b * num_kv_heads + (num_kv_heads - 1 - h)) * head_dim;", 1),
+    ("append_k_only", APPEND, "v_pages[dst + d] = v_new[src + d];", "", 1),
 ]
 
 
@@ -83,7 +89,7 @@ def test_pins_catch_mutant(tmp_path, mid, func, old, new, count):
     path.write_text(mutate(src, func, old, new, count))
     lib = oracle.compile_library(path, tmp_path / f"lib{mid}.so")
     orc = oracle.Oracle(lib)
-    pins = ATTENTION_PINS if func == ATT else STAGE_PINS
+    pins = {ATT: ATTENTION_PINS, APPEND: APPEND_PINS}.get(func, STAGE_PINS)
     caught = []
     for pin in pins:
         try:
