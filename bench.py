@@ -267,6 +267,33 @@ def run_decode_loop(tensors, ev, stream):
         e2.record(stream)
 
 
+def time_append_step(batch, tensors, steps, warmup, stream):
+    """The whole decode step of one layer, decode_attention_append: write the new
+    token's K/V for every trajectory, then attend (2 launches)."""
+    q, k, v, bt, cl, out, lse, ws = tensors
+    w = batch.workload
+    g = torch.Generator(device=q.device).manual_seed(w.seed + 7)
+    k_new = torch.randn((q.shape[0], w.num_kv_heads, w.head_dim), generator=g,
+                        device=q.device).to(torch.bfloat16)
+    v_new = torch.randn_like(k_new, dtype=torch.float32).to(torch.bfloat16)
+    for _ in range(warmup):
+        cadkv.decode_attention_append(q, k_new, v_new, k, v, bt, cl, out=out, lse=lse,
+                                      workspace=ws, stream=stream)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        cadkv.decode_attention_append(q, k_new, v_new, k, v, bt, cl, out=out, lse=lse,
+                                      workspace=ws, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    nbytes = decode_bytes(batch.context_lens, w.num_q_heads, w.num_kv_heads, w.head_dim)
+    nbytes += 2 * 2 * k_new.numel() * 2          # read k_new, v_new; write them to the pool
+    return {"gbps": round(nbytes / (ms * 1e-3) / 1e9, 1), "ms_per_step": round(ms, 4),
+            "steps_per_s": round(1e3 / ms, 1), "launches_per_step": 2,
+            "status": cadkv.decode_attention_status(ws)}
+
+
 def e2e_loop(batch, tensors, steps, warmup, stream):
     """decode_attention through the C ABI with host inputs and outputs: every
     step copies q, block_table and context_lens from pinned host memory, runs
@@ -521,6 +548,7 @@ def main():
     all_bytes = sum_over_ranks(float(nbytes), world)
     value = all_bytes * args.steps / (total_ms * 1e-3) / 1e9
 
+    append = time_append_step(batch, tensors, max(args.steps // 4, 20), 3, stream)
     e2e_s, h2d, d2h = e2e_loop(batch, tensors, max(args.steps // 4, 20), 3, stream)
     e2e_s = max_over_ranks(e2e_s, world)
     e2e_value = all_bytes / e2e_s / 1e9
@@ -556,7 +584,7 @@ def main():
         "e2e": {"value": round(e2e_value, 1), "unit": "GB/s",
                 "ms_per_step": round(e2e_s * 1e3, 4),
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": 2 * args.steps,
+        "gpu_launches": 2 * args.steps,  # plan + attention per timed step
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(achieved / peak, 4),
                      "peak_kind": kind, "kernel": "decode_attention_kernel<128>",
@@ -564,6 +592,7 @@ def main():
                      "read_probe_gbps": round(read_gbps, 1),
                      "frac_of_read_probe": round(achieved / read_gbps, 4),
                      "traffic": profiled_traffic(PROFILE_SUMMARY, KERNEL_SOURCE)},
+        "decode_step_with_append": append,
         "clocks": clocks,
         "device_status": status,
     }

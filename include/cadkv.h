@@ -183,6 +183,26 @@ int decode_attention_run(const void *q, const void *k_pages, const void *v_pages
                          size_t workspace_bytes, cadkv_stream_t stream);
 
 /*
+ * The whole decode step of one layer: first append each trajectory's new-token
+ * key and value, then attend.  n_b = context_lens[b] counts the new token, so
+ * k_new[b][h][:] and v_new[b][h][:] (bf16 [batch][num_kv_heads][head_dim]) are
+ * written to token position n_b - 1 -- page block_table[b][(n_b - 1) / 16],
+ * slot (n_b - 1) % 16 -- of k_pages / v_pages, which are modified in place;
+ * trajectories with n_b = 0 append nothing.  Then exactly decode_attention
+ * over the updated pages.  The append runs in extra CTAs of the planner
+ * launch, so the step is still two launches.  (Sec. 2.3: every decode step
+ * extends each trajectory's KV cache by one token before attending over it.)
+ * A bad last page is reported as CADKV_ERR_OOB in the status word, and the
+ * row is not written.
+ */
+int decode_attention_append(const void *q, const void *k_new, const void *v_new,
+                            void *k_pages, void *v_pages, const int32_t *block_table,
+                            const int32_t *context_lens, void *out, float *lse, int batch,
+                            int num_q_heads, int num_kv_heads, int head_dim, int page_size,
+                            int num_pages, int max_pages, void *workspace,
+                            size_t workspace_bytes, cadkv_stream_t stream);
+
+/*
  * Synchronise `stream` and return the device status word the last call that
  * used `workspace` left (CADKV_OK, CADKV_ERR_SHAPE, CADKV_ERR_OOB or
  * CADKV_ERR_TIMEOUT), or CADKV_ERR_CUDA if the copy failed.

@@ -57,6 +57,8 @@ _SIGNATURES = {
     "decode_attention_run": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I,
                                   _P, _SZ, _P]),
     "decode_attention_status": (_I, [_P, _P]),
+    "decode_attention_append": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I,
+                                     _I, _I, _P, _SZ, _P]),
     "decode_attention_noalloc": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I,
                                       _P]),
     "kv_prefix_stage_workspace_size": (_SZ, [_I]),
@@ -189,6 +191,27 @@ def decode_attention(q, k_pages, v_pages, block_table, context_lens, out=None, l
         _ptr(out), _ptr(lse), batch, hq, hkv, d, page, num_pages, max_pages,
         int(slice_pages), _ptr(workspace), workspace.numel(), _stream(stream, q.device))
     _check("decode_attention", rc)
+    return out, lse
+
+
+def decode_attention_append(q, k_new, v_new, k_pages, v_pages, block_table, context_lens,
+                            out=None, lse=None, workspace=None, want_lse: bool = True,
+                            stream=None):
+    """The decode step: write the new token's K/V (bf16 [B, Hkv, D]) at position
+    n_b - 1 of each trajectory's pages (in place), then attend; returns (out, lse)."""
+    batch, hq, hkv, d, page, num_pages, max_pages = _decode_args(
+        q, k_pages, v_pages, block_table, context_lens)
+    for name, t in (("k_new", k_new), ("v_new", v_new)):
+        _need(t, name, torch.bfloat16, 3, q.device)
+        if tuple(t.shape) != (batch, hkv, d):
+            raise ValueError(f"{name} must be [B, Hkv, D]")
+    out, lse, workspace = _outputs(q, out, lse, want_lse, workspace, batch, hq, hkv, d,
+                                   max_pages)
+    rc = library().decode_attention_append(
+        _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_pages), _ptr(v_pages), _ptr(block_table),
+        _ptr(context_lens), _ptr(out), _ptr(lse), batch, hq, hkv, d, page, num_pages,
+        max_pages, _ptr(workspace), workspace.numel(), _stream(stream, q.device))
+    _check("decode_attention_append", rc)
     return out, lse
 
 

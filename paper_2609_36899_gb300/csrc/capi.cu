@@ -142,8 +142,16 @@ int workspace_carve(const DecodeShape &s, void *workspace, size_t workspace_byte
     return CADKV_OK;
 }
 
+// New-token rows written into the pool before attention (decode_attention_append).
+struct AppendArgs {
+    const void *k_new, *v_new;
+    void *k_pages, *v_pages;
+    const int32_t *block_table;
+};
+
 int plan_impl(const int32_t *context_lens, void *out, float *lse, const DecodeShape &s,
-              int slice_pages, void *workspace, size_t workspace_bytes, cudaStream_t stream)
+              int slice_pages, void *workspace, size_t workspace_bytes, cudaStream_t stream,
+              const AppendArgs *append = nullptr)
 {
     int rc = check_decode_shape(s);
     if (rc != CADKV_OK)
@@ -178,6 +186,14 @@ int plan_impl(const int32_t *context_lens, void *out, float *lse, const DecodeSh
     p.max_pages = s.max_pages;
     p.slice_cap = L.slice_cap;
     p.slice_pages = slice_pages;
+    if (append) {
+        p.k_new = static_cast<const __nv_bfloat16 *>(append->k_new);
+        p.v_new = static_cast<const __nv_bfloat16 *>(append->v_new);
+        p.k_pages = static_cast<__nv_bfloat16 *>(append->k_pages);
+        p.v_pages = static_cast<__nv_bfloat16 *>(append->v_pages);
+        p.block_table = append->block_table;
+        p.num_pages = s.num_pages;
+    }
     return launch_plan(p, stream) == cudaSuccess ? CADKV_OK : CADKV_ERR_CUDA;
 }
 
@@ -520,6 +536,33 @@ int decode_attention(const void *q, const void *k_pages, const void *v_pages,
 int decode_attention_status(const void *workspace, cadkv_stream_t stream)
 {
     return read_status(workspace, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int decode_attention_append(const void *q, const void *k_new, const void *v_new, void *k_pages,
+                            void *v_pages, const int32_t *block_table,
+                            const int32_t *context_lens, void *out, float *lse, int batch,
+                            int num_q_heads, int num_kv_heads, int head_dim, int page_size,
+                            int num_pages, int max_pages, void *workspace,
+                            size_t workspace_bytes, cadkv_stream_t stream)
+{
+    const DecodeShape s{batch, num_q_heads, num_kv_heads, head_dim, page_size, num_pages, max_pages};
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int rc = check_decode_shape(s);
+    if (rc != CADKV_OK)
+        return rc;
+    if (batch == 0)
+        return CADKV_OK;
+    rc = check_run_args(q, k_pages, v_pages, block_table, context_lens, out, lse, s);
+    if (rc != CADKV_OK)
+        return rc;
+    if (!k_new || !v_new || !aligned(k_new, 16) || !aligned(v_new, 16))
+        return CADKV_ERR_INVALID;
+    const AppendArgs append{k_new, v_new, k_pages, v_pages, block_table};
+    rc = plan_impl(context_lens, out, lse, s, 0, workspace, workspace_bytes, st, &append);
+    if (rc != CADKV_OK)
+        return rc;
+    return run_impl(q, k_pages, v_pages, block_table, context_lens, out, lse, s, workspace,
+                    workspace_bytes, st);
 }
 
 }  // extern "C"

@@ -47,8 +47,41 @@ __host__ __device__ constexpr size_t align_up(size_t x, size_t a) { return (x + 
 
 // ------------------------------------------------------------------ planner
 
+// CTAs 1.. of the planner launch: write each trajectory's new-token K and V
+// rows into slot (n_b - 1) % 16 of page block_table[b][(n_b - 1) / 16].  One
+// warp per (trajectory, KV head); lanes 0-15 copy K, lanes 16-31 copy V, 16
+// bytes each.  Invalid lengths or pages are skipped here: CTA 0 flags bad
+// lengths, and the attention kernel flags the bad page when it reads it.
+__device__ __forceinline__ void append_rows(const PlanParams &p)
+{
+    const int lane = threadIdx.x & 31;
+    const int row = (blockIdx.x - 1) * kAppendRowsPerCta + (threadIdx.x >> 5);
+    if (row >= p.batch * p.num_kv_heads)
+        return;
+    const int b = row / p.num_kv_heads, g = row % p.num_kv_heads;
+    const int n = p.context_lens[b];
+    if (n < 1 || n > p.max_pages * kPageSize)
+        return;
+    const int phys = p.block_table[(size_t)b * p.max_pages + (n - 1) / kPageSize];
+    if (phys < 0 || phys >= p.num_pages)
+        return;
+    const int slot = (n - 1) % kPageSize;
+    const bool is_v = lane >= 16;
+    const uint4 *src = reinterpret_cast<const uint4 *>((is_v ? p.v_new : p.k_new) +
+                                                       (size_t)row * p.head_dim);
+    uint4 *dst = reinterpret_cast<uint4 *>(
+        (is_v ? p.v_pages : p.k_pages) +
+        (((size_t)phys * p.num_kv_heads + g) * kPageSize + slot) * p.head_dim);
+    for (int c = lane & 15; c < p.head_dim / 8; c += 16)
+        dst[c] = src[c];
+}
+
 __global__ void __launch_bounds__(1024, 1) plan_kernel(const PlanParams p)
 {
+    if (blockIdx.x > 0) {
+        append_rows(p);
+        return;
+    }
     __shared__ long long warp_sums[32];
     __shared__ long long carry_s;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -717,7 +750,9 @@ DecodeWorkspaceLayout decode_workspace_layout(int batch, int num_kv_heads, int g
 
 cudaError_t launch_plan(const PlanParams &p, cudaStream_t stream)
 {
-    plan_kernel<<<1, 1024, 0, stream>>>(p);
+    const int append_ctas =
+        p.k_new ? (p.batch * p.num_kv_heads + kAppendRowsPerCta - 1) / kAppendRowsPerCta : 0;
+    plan_kernel<<<1 + append_ctas, 1024, 0, stream>>>(p);
     return cudaGetLastError();
 }
 

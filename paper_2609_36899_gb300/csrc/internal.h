@@ -54,7 +54,15 @@ struct PlanParams {
     int batch, num_q_heads, num_kv_heads, head_dim, max_pages;
     int slice_cap;      // upper bound on slices (partial capacity)
     int slice_pages;    // forced slice length in pages, 0 = automatic
+    // Optional fused KV append (CTAs 1.. of the planner launch): the new
+    // token's rows k_new/v_new [batch][Hkv][D] go to position n_b - 1.
+    const __nv_bfloat16 *k_new, *v_new;  // null: no append
+    __nv_bfloat16 *k_pages, *v_pages;
+    const int *block_table;
+    int num_pages;
 };
+
+constexpr int kAppendRowsPerCta = 32;  // one warp per (trajectory, KV head)
 
 struct AttnParams {
     const __nv_bfloat16 *q;
@@ -72,7 +80,7 @@ struct AttnParams {
     float scale_log2;    // log2(e) / sqrt(D)
 };
 
-cudaError_t launch_plan(const PlanParams &p, cudaStream_t stream);
+cudaError_t launch_plan(const PlanParams &p, cudaStream_t stream);  // + append CTAs if k_new
 cudaError_t launch_attention(const AttnParams &p, const CUtensorMap &kmap,
                              const CUtensorMap &vmap, int head_dim, int grid,
                              cudaStream_t stream);
