@@ -22,6 +22,9 @@ Definitions (written out in ``oracle.c``):
   staged prefix into a paged pool (Sec. 4.4, phase 3).
 * ``kv_append`` -- the write of each trajectory's new-token key and value
   into its paged cache that precedes attention in every decode step.
+* ``prefill_attention`` -- chunked (re-)prefill attention: each trajectory's
+  last C_b tokens attend causally over its paged KV (the fallback of Sec. 4.4
+  when prepared KV state cannot be used).
 
 Every function is pinned by the CPU tests in ``tests/test_oracle_*.py``.
 """
@@ -102,6 +105,10 @@ class Oracle:
         f.restype = ctypes.c_int
         f.argtypes = [_P, _P, _I64, _I64, _I64, _I64, _I64, _P, _I64, _P, _I64,
                       _I64, _I64, _P, _P]
+        f = self.lib.oracle_prefill_attention
+        f.restype = ctypes.c_int
+        f.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64, _I64, _I64,
+                      _P, _P, ctypes.c_int]
         f = self.lib.oracle_kv_append
         f.restype = ctypes.c_int
         f.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64, _I64]
@@ -217,6 +224,30 @@ class Oracle:
         self._check(rc)
         return k_pages, v_pages
 
+    def prefill_attention(self, q, q_offsets, k_pages, v_pages, block_table, context_lens,
+                          num_threads: int = 0):
+        """Causal attention of each trajectory's last C_b tokens.
+
+        q: uint16 [T, Hq, D] (T = q_offsets[-1]); q_offsets: int64 [B + 1].
+        Returns (out float64 [T, Hq, D], lse float64 [T, Hq]).
+        """
+        q, k_pages, v_pages = _u16(q), _u16(k_pages), _u16(v_pages)
+        q_offsets = np.ascontiguousarray(q_offsets, dtype=np.int64)
+        block_table, context_lens = _i32(block_table), _i32(context_lens)
+        total, hq, d = q.shape
+        num_pages, hkv, page, d2 = k_pages.shape
+        batch = context_lens.shape[0]
+        if d2 != d or q_offsets.shape != (batch + 1,) or q_offsets[-1] != total:
+            raise ValueError("inconsistent prefill shapes")
+        out = np.empty((total, hq, d), dtype=np.float64)
+        lse = np.empty((total, hq), dtype=np.float64)
+        rc = self.lib.oracle_prefill_attention(
+            _ptr(q), _ptr(q_offsets), _ptr(k_pages), _ptr(v_pages), _ptr(block_table),
+            _ptr(context_lens), batch, hq, hkv, d, page, num_pages, block_table.shape[1],
+            _ptr(out), _ptr(lse), int(num_threads))
+        self._check(rc)
+        return out, lse
+
 
 _DEFAULT: Oracle | None = None
 
@@ -242,3 +273,7 @@ def prefix_load(*args, **kwargs):
 
 def kv_append(*args, **kwargs):
     return default().kv_append(*args, **kwargs)
+
+
+def prefill_attention(*args, **kwargs):
+    return default().prefill_attention(*args, **kwargs)

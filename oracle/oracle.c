@@ -54,6 +54,19 @@
  *    token position n_b - 1, i.e. page block_table[b][(n_b - 1) / P], slot
  *    (n_b - 1) % P.  Trajectories with n_b = 0 append nothing.
  *
+ * 5. oracle_prefill_attention: chunked prefill (re-prefill) attention over the
+ *    paged pool -- the fallback of Sec. 4.4 when prepared KV state cannot be
+ *    used and the destination recomputes the prefix.  Trajectory b contributes
+ *    its last C_b = q_offsets[b+1] - q_offsets[b] tokens as queries; their K
+ *    and V are already in the pool, so query i of b sits at absolute position
+ *    p = n_b - C_b + i and attends causally to keys t = 0 .. p:
+ *
+ *        s_t = (q_{row,h} . K_t) / sqrt(D)   for t <= p
+ *        out[row,h,:] = sum_{t<=p} exp(s_t - m) V_t / sum_{t<=p} exp(s_t - m)
+ *        lse[row,h]   = m + ln sum_{t<=p} exp(s_t - m)
+ *
+ *    with row = q_offsets[b] + i, g = h / G as above.  Requires C_b <= n_b.
+ *
  * Pool layout: per layer, K and V are each [num_pages][Hkv][P][D] bf16
  * (head-major inside a page); layers are stacked with stride
  * num_pages * Hkv * P * D elements.
@@ -336,6 +349,85 @@ int oracle_kv_append(uint16_t *k_pages, uint16_t *v_pages, const uint16_t *k_new
                 v_pages[dst + d] = v_new[src + d];
             }
         }
+    }
+    return 0;
+}
+
+/*
+ * q: [T][Hq][D] bf16 bits, T = q_offsets[batch]; out: [T][Hq][D]; lse: [T][Hq].
+ */
+int oracle_prefill_attention(const uint16_t *q, const int64_t *q_offsets,
+                             const uint16_t *k_pages, const uint16_t *v_pages,
+                             const int32_t *block_table, const int32_t *context_lens,
+                             int64_t batch, int64_t num_q_heads, int64_t num_kv_heads,
+                             int64_t head_dim, int64_t page_size, int64_t num_pages,
+                             int64_t max_pages, double *out, double *lse, int num_threads)
+{
+    if (!q || !q_offsets || !k_pages || !v_pages || !block_table || !context_lens || !out ||
+        !lse)
+        return -1;
+    if (batch < 0 || num_q_heads <= 0 || num_kv_heads <= 0 || head_dim <= 0 ||
+        page_size <= 0 || num_q_heads % num_kv_heads != 0)
+        return -1;
+    int rc = check_lengths(block_table, context_lens, batch, page_size, num_pages,
+                           max_pages);
+    if (rc != 0)
+        return rc;
+    if (q_offsets[0] != 0)
+        return -1;
+    for (int64_t b = 0; b < batch; ++b) {
+        const int64_t chunk = q_offsets[b + 1] - q_offsets[b];
+        if (chunk < 0 || chunk > context_lens[b])
+            return -2;
+    }
+    const int64_t total = q_offsets[batch];
+    const int64_t group = num_q_heads / num_kv_heads;
+    const double scale = 1.0 / sqrt((double)head_dim);
+    set_threads(num_threads);
+
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t i = 0; i < total * num_q_heads; ++i) {
+        const int64_t row = i / num_q_heads;
+        const int64_t h = i % num_q_heads;
+        int64_t b = 0;
+        while (q_offsets[b + 1] <= row)
+            ++b;
+        const int64_t chunk = q_offsets[b + 1] - q_offsets[b];
+        const int64_t pos = context_lens[b] - chunk + (row - q_offsets[b]);
+        const int64_t n = pos + 1;                /* keys 0 .. pos */
+        const int64_t g = h / group;
+        const uint16_t *qv = q + (row * num_q_heads + h) * head_dim;
+        double *o = out + i * head_dim;
+        double *s = (double *)malloc((size_t)n * sizeof(double));
+
+        double m = -INFINITY;
+        for (int64_t t = 0; t < n; ++t) {
+            const int64_t phys = block_table[b * max_pages + t / page_size];
+            const uint16_t *kv =
+                k_pages + ((phys * num_kv_heads + g) * page_size + t % page_size) * head_dim;
+            double dot = 0.0;
+            for (int64_t d = 0; d < head_dim; ++d)
+                dot += widen_bf16(qv[d]) * widen_bf16(kv[d]);
+            s[t] = dot * scale;
+            if (s[t] > m)
+                m = s[t];
+        }
+        for (int64_t d = 0; d < head_dim; ++d)
+            o[d] = 0.0;
+        double l = 0.0;
+        for (int64_t t = 0; t < n; ++t) {
+            const int64_t phys = block_table[b * max_pages + t / page_size];
+            const uint16_t *vv =
+                v_pages + ((phys * num_kv_heads + g) * page_size + t % page_size) * head_dim;
+            const double w = exp(s[t] - m);
+            l += w;
+            for (int64_t d = 0; d < head_dim; ++d)
+                o[d] += w * widen_bf16(vv[d]);
+        }
+        for (int64_t d = 0; d < head_dim; ++d)
+            o[d] /= l;
+        lse[i] = m + log(l);
+        free(s);
     }
     return 0;
 }

@@ -462,3 +462,75 @@ def pin_append_writes_only_the_new_slot(orc):
 
 
 APPEND_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_append_")]
+
+
+# --------------------------------------------------------------------------
+# chunked prefill attention
+# --------------------------------------------------------------------------
+
+def _prefill_case(seed, lens, chunks, hq, hkv, d):
+    rng = _rng(seed)
+    ks = [to_bf16_bits(rng.normal(size=(n, hkv, d))) for n in lens]
+    vs = [to_bf16_bits(rng.normal(size=(n, hkv, d))) for n in lens]
+    used = sum(-(-n // 16) for n in lens)
+    perm = rng.permutation(used + 2)
+    kp, table, cl = paged(ks, 16, perm, used + 2, fill=NAN_BF16)
+    vp, _, _ = paged(vs, 16, perm, used + 2, fill=NAN_BF16)
+    offs = np.concatenate([[0], np.cumsum(chunks)]).astype(np.int64)
+    q = to_bf16_bits(rng.normal(size=(int(offs[-1]), hq, d)))
+    return q, offs, kp, vp, table, cl, ks, vs
+
+
+def pin_prefill_matches_scipy_causal(orc):
+    """Chunk = whole context: causal self-attention, checked row by row with
+    scipy softmax over the keys at or before each query's position."""
+    lens, chunks = [37, 20], [37, 9]
+    hq, hkv, d = 4, 2, 64
+    q, offs, kp, vp, table, cl, ks, vs = _prefill_case(60, lens, chunks, hq, hkv, d)
+    out, lse = orc.prefill_attention(q, offs, kp, vp, table, cl)
+    for b, (n, c) in enumerate(zip(lens, chunks)):
+        for i in range(c):
+            pos = n - c + i
+            row = offs[b] + i
+            for h in range(hq):
+                kf = bits_to_f64(ks[b][:pos + 1, h // 2])
+                vf = bits_to_f64(vs[b][:pos + 1, h // 2])
+                s = kf @ bits_to_f64(q[row, h]) / math.sqrt(d)
+                np.testing.assert_allclose(out[row, h], sp.softmax(s) @ vf, rtol=1e-11, atol=1e-12)
+                assert abs(lse[row, h] - sp.logsumexp(s)) <= 1e-12 * max(1, abs(lse[row, h]))
+
+
+def pin_prefill_rows_equal_decode_at_their_position(orc):
+    """Each prefill row equals decode attention with the trajectory truncated
+    to that query's position (same bits)."""
+    lens, chunks = [50, 17, 33], [5, 0, 3]
+    hq, hkv, d = 8, 2, 64
+    q, offs, kp, vp, table, cl, _, _ = _prefill_case(61, lens, chunks, hq, hkv, d)
+    out, lse = orc.prefill_attention(q, offs, kp, vp, table, cl)
+    rows_b, rows_len = [], []
+    for b, (n, c) in enumerate(zip(lens, chunks)):
+        for i in range(c):
+            rows_b.append(b)
+            rows_len.append(n - c + i + 1)
+    dec_out, dec_lse = orc.decode_attention(q, kp, vp, table[rows_b],
+                                            np.array(rows_len, dtype=np.int32))
+    np.testing.assert_array_equal(out, dec_out)
+    np.testing.assert_array_equal(lse, dec_lse)
+
+
+def pin_prefill_is_causal(orc):
+    """Changing the last token's K and V changes only the last query row."""
+    lens, chunks = [40], [6]
+    q, offs, kp, vp, table, cl, ks, vs = _prefill_case(62, lens, chunks, 2, 1, 64)
+    a = orc.prefill_attention(q, offs, kp, vp, table, cl)
+    t = 39
+    ph, sl = table[0, t // 16], t % 16
+    kp2, vp2 = kp.copy(), vp.copy()
+    kp2[ph, :, sl] = to_bf16_bits(np.full((1, 64), 3.0))
+    vp2[ph, :, sl] = to_bf16_bits(np.full((1, 64), -5.0))
+    b_ = orc.prefill_attention(q, offs, kp2, vp2, table, cl)
+    np.testing.assert_array_equal(a[0][:5], b_[0][:5])
+    assert not np.allclose(a[0][5], b_[0][5])
+
+
+PREFILL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_prefill_")]

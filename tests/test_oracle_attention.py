@@ -46,3 +46,11 @@ from _pins import APPEND_PINS  # noqa: E402
 @pytest.mark.parametrize("pin", APPEND_PINS, ids=lambda f: f.__name__)
 def test_append_pin(orc, pin):
     pin(orc)
+
+
+from _pins import PREFILL_PINS  # noqa: E402
+
+
+@pytest.mark.parametrize("pin", PREFILL_PINS, ids=lambda f: f.__name__)
+def test_prefill_pin(orc, pin):
+    pin(orc)

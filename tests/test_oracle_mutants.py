@@ -15,12 +15,13 @@ import re
 import pytest
 
 import oracle
-from _pins import APPEND_PINS, ATTENTION_PINS, STAGE_PINS
+from _pins import APPEND_PINS, ATTENTION_PINS, PREFILL_PINS, STAGE_PINS
 
 ATT = "oracle_decode_attention"
 STAGE = "oracle_prefix_stage"
 LOAD = "oracle_prefix_load"
 APPEND = "oracle_kv_append"
+PREFILL = "oracle_prefill_attention"
 
 MUTANTS = [
     # (id, function, old, new, count) -- count 0 replaces every occurrence
@@ -64,6 +65,15 @@ MUTANTS = [
      "const int64_t src = (b * num_kv_heads + h) * head_dim;",
      "const int64_t src = (b * num_kv_heads + (num_kv_heads - 1 - h)) * head_dim;", 1),
     ("append_k_only", APPEND, "v_pages[dst + d] = v_new[src + d];", "", 1),
+    ("prefill_excludes_own_token", PREFILL, "const int64_t n = pos + 1;",
+     "const int64_t n = pos > 0 ? pos : 1;", 1),
+    ("prefill_attends_whole_context", PREFILL, "const int64_t n = pos + 1;",
+     "const int64_t n = context_lens[b];", 1),
+    ("prefill_chunk_at_start", PREFILL,
+     "const int64_t pos = context_lens[b] - chunk + (row - q_offsets[b]);",
+     "const int64_t pos = row - q_offsets[b];", 1),
+    ("prefill_gqa_interleaved", PREFILL, "const int64_t g = h / group;",
+     "const int64_t g = h % num_kv_heads;", 1),
 ]
 
 
@@ -89,7 +99,8 @@ def test_pins_catch_mutant(tmp_path, mid, func, old, new, count):
     path.write_text(mutate(src, func, old, new, count))
     lib = oracle.compile_library(path, tmp_path / f"lib{mid}.so")
     orc = oracle.Oracle(lib)
-    pins = {ATT: ATTENTION_PINS, APPEND: APPEND_PINS}.get(func, STAGE_PINS)
+    pins = {ATT: ATTENTION_PINS, APPEND: APPEND_PINS, PREFILL: PREFILL_PINS}.get(
+        func, STAGE_PINS)
     caught = []
     for pin in pins:
         try:
