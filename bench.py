@@ -443,6 +443,54 @@ def bench_landscape(device, steps, warmup, batches=(8, 32, 128, 512),
     return cells
 
 
+def bench_prefill(device, steps, warmup, batch=8, context=16384, chunk=512, hq=32, hkv=8):
+    """Chunked re-prefill: each of `batch` trajectories recomputes attention for
+    its last `chunk` tokens over a `context`-token paged KV (32/8 heads, D=128)."""
+    from paper_2609_36899_gb300.workloads import DecodeWorkload
+    w = DecodeWorkload("prefill", batch, hq, hkv, 128, "fixed", tuple([context] * batch),
+                       context, 20267)
+    b = make_decode_batch(w, device=device)
+    offs = torch.arange(0, (batch + 1) * chunk, chunk, dtype=torch.int64, device=device)
+    g = torch.Generator(device=device).manual_seed(20268)
+    q = torch.randn((batch * chunk, hq, 128), generator=g, device=device).to(torch.bfloat16)
+    bt = torch.from_numpy(b.block_table).to(device)
+    cl = torch.from_numpy(b.context_lens).to(device)
+    out = torch.empty_like(q)
+    lse = torch.empty((batch * chunk, hq), dtype=torch.float32, device=device)
+    ws = torch.empty(max(int(cadkv.library().prefill_attention_workspace_size(batch)), 1),
+                     dtype=torch.uint8, device=device)
+    stream = torch.cuda.current_stream(device)
+    for _ in range(warmup):
+        cadkv.prefill_attention(q, offs, b.k_pages, b.v_pages, bt, cl, out=out, lse=lse,
+                                workspace=ws, stream=stream)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        cadkv.prefill_attention(q, offs, b.k_pages, b.v_pages, bt, cl, out=out, lse=lse,
+                                workspace=ws, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    # algorithmic flops: each (row, head) at position p does 2 D (p + 1) for QK^T and for PV
+    pos = np.arange(context - chunk, context, dtype=np.float64)
+    flops = batch * hq * float((4.0 * 128 * (pos + 1)).sum())
+    try:
+        peak = float(json.load(open(PEAKS_FILE))["bf16_tflops"])
+        kind = "measured"
+    except Exception:
+        peak, kind = 1900.0, "fallback"
+    tflops = flops / (ms * 1e-3) / 1e12
+    res = {"workload": f"chunked prefill: {batch} trajectories x last {chunk} of {context} "
+                       f"tokens, {hq}/{hkv} heads, D=128, causal",
+           "ms_per_call": round(ms, 4), "tflops": round(tflops, 1),
+           "status": cadkv.prefill_attention_status(ws), "launches_per_call": 2,
+           "roofline": {"bound": "tensor", "achieved": round(tflops, 1), "peak": peak,
+                        "unit": "TFLOP/s", "frac": round(tflops / peak, 4), "peak_kind": kind}}
+    del b, q, out
+    torch.cuda.empty_cache()
+    return res
+
+
 def bench_config(name, device, steps, warmup):
     w = DECODE_WORKLOADS[name]
     batch = make_decode_batch(w, device=device)
@@ -487,7 +535,8 @@ def main():
     ap.add_argument("--steps", type=int, default=400)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=sorted(DECODE_WORKLOADS) + ["staging", "landscape"],
+    ap.add_argument("--workload",
+                    choices=sorted(DECODE_WORKLOADS) + ["staging", "landscape", "prefill"],
                     default="mixed",
                     help="decode workload of the headline line, or 'staging' to time "
                          "only prefix staging")
@@ -513,6 +562,11 @@ def main():
     if args.workload == "staging":
         res = bench_staging(device, reps=args.steps, layers=args.staging_layers,
                             batch=args.staging_batch)
+        if rank == 0:
+            print(json.dumps(res), flush=True)
+        return
+    if args.workload == "prefill":
+        res = bench_prefill(device, args.steps, args.warmup)
         if rank == 0:
             print(json.dumps(res), flush=True)
         return

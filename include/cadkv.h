@@ -210,6 +210,43 @@ int decode_attention_append(const void *q, const void *k_new, const void *v_new,
 int decode_attention_status(const void *workspace, cadkv_stream_t stream);
 
 /* ------------------------------------------------------------------------ */
+/* Chunked (re-)prefill attention (Sec. 4.4: the fallback when prepared KV   */
+/* state cannot be used and the destination recomputes the prefix)           */
+/* ------------------------------------------------------------------------ */
+
+/* Bytes of workspace prefill_attention needs for `batch` trajectories. */
+size_t prefill_attention_workspace_size(int batch);
+
+/*
+ * Causal attention of each trajectory's last C_b tokens over its paged KV.
+ *   q          bf16 [total_q][num_q_heads][head_dim]; trajectory b owns rows
+ *              q_offsets[b] .. q_offsets[b+1]-1 (C_b of them)
+ *   q_offsets  device int64 [batch + 1], q_offsets[0] = 0, non-decreasing,
+ *              q_offsets[batch] = total_q
+ *   k_pages, v_pages, block_table, context_lens: as decode_attention; the K/V
+ *              of the C_b query tokens are already in the pool, at positions
+ *              n_b - C_b .. n_b - 1 (so C_b <= n_b)
+ *   out        bf16 [total_q][num_q_heads][head_dim]
+ *   lse        fp32 [total_q][num_q_heads] or NULL
+ * Query row i of trajectory b sits at position p = n_b - C_b + i and attends
+ * to keys 0 .. p:  out = softmax_t<=p(q . K_t / sqrt(D)) V,  lse = ln sum exp.
+ * Runs on the tcgen05 tensor cores (accumulators in TMEM), one CTA per
+ * (trajectory, KV head, tile of 128 (query token, head) rows).
+ * Supported: head_dim 128, page_size 16, G = Hq / Hkv in {1, 2, 4, 8}.
+ * A trajectory with C_b > n_b or n_b out of range is skipped (its rows are
+ * not written) and CADKV_ERR_SHAPE lands in the status word.
+ */
+int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pages,
+                      const void *v_pages, const int32_t *block_table,
+                      const int32_t *context_lens, void *out, float *lse, int batch,
+                      int total_q, int num_q_heads, int num_kv_heads, int head_dim,
+                      int page_size, int num_pages, int max_pages, void *workspace,
+                      size_t workspace_bytes, cadkv_stream_t stream);
+
+/* As decode_attention_status, for a prefill workspace. */
+int prefill_attention_status(const void *workspace, cadkv_stream_t stream);
+
+/* ------------------------------------------------------------------------ */
 /* Prefix staging (Sec. 4.4, phase 1) and its inverse (Sec. 4.4, phase 3)    */
 /* ------------------------------------------------------------------------ */
 

@@ -66,6 +66,10 @@ _SIGNATURES = {
     "kv_prefix_load": (_I, [_P, _P, _I, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
     "kv_prefix_stage_status": (_I, [_P, _P]),
     "cadkv_hbm_read_probe": (_I, [_P, _SZ, _P, _P]),
+    "prefill_attention_workspace_size": (_SZ, [_I]),
+    "prefill_attention": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I,
+                               _P, _SZ, _P]),
+    "prefill_attention_status": (_I, [_P, _P]),
 }
 
 _lib = None
@@ -261,6 +265,45 @@ def decode_attention_noalloc(q, k_pages, v_pages, block_table, context_lens, out
         _stream(stream, q.device))
     _check("decode_attention_noalloc", rc)
     return out, lse
+
+
+def prefill_attention(q, q_offsets, k_pages, v_pages, block_table, context_lens, out=None,
+                      lse=None, workspace=None, want_lse: bool = True, stream=None):
+    """Causal attention of each trajectory's last C_b tokens over its paged KV.
+
+    q bf16 [T, Hq, D]; q_offsets int64 [B + 1] (device); the rest as in
+    decode_attention.  Returns (out [T, Hq, D], lse [T, Hq]).
+    """
+    _need(q, "q", torch.bfloat16, 3)
+    dev = q.device
+    _need(q_offsets, "q_offsets", torch.int64, 1, dev)
+    _need(k_pages, "k_pages", torch.bfloat16, 4, dev)
+    _need(v_pages, "v_pages", torch.bfloat16, 4, dev)
+    _need(block_table, "block_table", torch.int32, 2, dev)
+    _need(context_lens, "context_lens", torch.int32, 1, dev)
+    total, hq, d = q.shape
+    num_pages, hkv, page, d2 = k_pages.shape
+    batch = context_lens.shape[0]
+    if v_pages.shape != k_pages.shape or d2 != d or q_offsets.shape[0] != batch + 1:
+        raise ValueError("inconsistent prefill shapes")
+    if out is None:
+        out = torch.empty_like(q)
+    if lse is None and want_lse:
+        lse = torch.empty((total, hq), dtype=torch.float32, device=dev)
+    if workspace is None:
+        workspace = torch.empty(max(int(library().prefill_attention_workspace_size(batch)), 1),
+                                dtype=torch.uint8, device=dev)
+    rc = library().prefill_attention(
+        _ptr(q), _ptr(q_offsets), _ptr(k_pages), _ptr(v_pages), _ptr(block_table),
+        _ptr(context_lens), _ptr(out), _ptr(lse), batch, total, hq, hkv, d, page, num_pages,
+        block_table.shape[1], _ptr(workspace), workspace.numel(), _stream(stream, dev))
+    _check("prefill_attention", rc)
+    return out, lse, workspace
+
+
+def prefill_attention_status(workspace, stream=None) -> int:
+    return int(library().prefill_attention_status(_ptr(workspace),
+                                                  _stream(stream, workspace.device)))
 
 
 # ------------------------------------------------------------------ pool + staging

@@ -19,7 +19,8 @@ CSRC = PKG / "csrc"
 INCLUDE = PKG.parent / "include"
 BUILD_DIR = PKG / "_build"
 LIBRARY = PKG / "libcadkv.so"
-SOURCES = ["capi.cu", "decode_attention.cu", "prefix_stage.cu", "hbm_probe.cu"]
+SOURCES = ["capi.cu", "decode_attention.cu", "prefix_stage.cu", "hbm_probe.cu",
+           "prefill_attention.cu"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC",

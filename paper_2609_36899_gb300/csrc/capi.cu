@@ -28,6 +28,8 @@ constexpr int kAbiVersion = (1 << 16) | 0;
 
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
+size_t align_up_host(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
 int device_sms()
 {
     static std::mutex mu;
@@ -534,6 +536,98 @@ int decode_attention(const void *q, const void *k_pages, const void *v_pages,
 }
 
 int decode_attention_status(const void *workspace, cadkv_stream_t stream)
+{
+    return read_status(workspace, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t prefill_attention_workspace_size(int batch)
+{
+    if (batch < 0)
+        return 0;
+    return align_up_host(sizeof(WorkspaceHeader), kWorkspaceAlign) +
+           align_up_host((size_t)(batch + 1) * sizeof(long long), kWorkspaceAlign);
+}
+
+int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pages,
+                      const void *v_pages, const int32_t *block_table,
+                      const int32_t *context_lens, void *out, float *lse, int batch,
+                      int total_q, int num_q_heads, int num_kv_heads, int head_dim,
+                      int page_size, int num_pages, int max_pages, void *workspace,
+                      size_t workspace_bytes, cadkv_stream_t stream)
+{
+    if (batch < 0 || total_q < 0 || num_q_heads <= 0 || num_kv_heads <= 0 || max_pages < 0 ||
+        num_pages <= 0 || num_q_heads % num_kv_heads != 0)
+        return CADKV_ERR_SHAPE;
+    const int group = num_q_heads / num_kv_heads;
+    if (head_dim != 128 || page_size != kPageSize ||
+        (group != 1 && group != 2 && group != 4 && group != 8))
+        return CADKV_ERR_UNSUPPORTED;
+    if ((long long)num_pages * num_kv_heads * kPageSize > INT32_MAX ||
+        (long long)max_pages * kPageSize > INT32_MAX)
+        return CADKV_ERR_UNSUPPORTED;
+    if (batch == 0 || total_q == 0)
+        return CADKV_OK;
+    if (!q || !q_offsets || !k_pages || !v_pages || !block_table || !context_lens || !out)
+        return CADKV_ERR_INVALID;
+    if (!aligned(q, 16) || !aligned(k_pages, 16) || !aligned(v_pages, 16) || !aligned(out, 16) ||
+        !aligned(q_offsets, 8) || !aligned(block_table, 4) || !aligned(context_lens, 4) ||
+        (lse && !aligned(lse, 4)))
+        return CADKV_ERR_INVALID;
+    if (!workspace || !aligned(workspace, kWorkspaceAlign) ||
+        workspace_bytes < prefill_attention_workspace_size(batch))
+        return CADKV_ERR_WORKSPACE;
+    EncodeTiledFn fn = encode_tiled_fn();
+    if (!fn)
+        return CADKV_ERR_CUDA;
+    // Q viewed as {D, Hq, T}: box {64, G, 128/G} = 128 rows (token-major, head-minor)
+    CUtensorMap qmap, kmap, vmap;
+    {
+        const cuuint64_t dims[3] = {(cuuint64_t)head_dim, (cuuint64_t)num_q_heads,
+                                    (cuuint64_t)total_q};
+        const cuuint64_t strides[2] = {(cuuint64_t)head_dim * 2,
+                                       (cuuint64_t)num_q_heads * head_dim * 2};
+        const cuuint32_t box[3] = {64, (cuuint32_t)group, (cuuint32_t)(128 / group)};
+        const cuuint32_t elem[3] = {1, 1, 1};
+        if (fn(&qmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(q), dims, strides, box,
+               elem, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return CADKV_ERR_CUDA;
+    }
+    int whole = 0;
+    if (encode_pages_map(&kmap, k_pages, num_pages, num_kv_heads, head_dim, false, &whole) !=
+            CADKV_OK ||
+        encode_pages_map(&vmap, v_pages, num_pages, num_kv_heads, head_dim, false, &whole) !=
+            CADKV_OK)
+        return CADKV_ERR_CUDA;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    PrefillParams p{};
+    p.q_offsets = reinterpret_cast<const long long *>(q_offsets);
+    p.context_lens = context_lens;
+    p.block_table = block_table;
+    p.out = static_cast<__nv_bfloat16 *>(out);
+    p.lse = lse;
+    p.hdr = reinterpret_cast<WorkspaceHeader *>(ws);
+    p.item_prefix = reinterpret_cast<long long *>(ws + align_up_host(sizeof(WorkspaceHeader),
+                                                                      kWorkspaceAlign));
+    p.total_q = total_q;
+    p.batch = batch;
+    p.num_q_heads = num_q_heads;
+    p.num_kv_heads = num_kv_heads;
+    p.group = group;
+    p.max_pages = max_pages;
+    p.num_pages = num_pages;
+    p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
+    // upper bound on work items: sum_b ceil(C_b G / 128) <= T G / 128 + B
+    const long long grid = (long long)num_kv_heads * (batch + ((long long)total_q * group + 127) / 128);
+    if (grid > INT32_MAX)
+        return CADKV_ERR_UNSUPPORTED;
+    return launch_prefill(p, qmap, kmap, vmap, (int)grid, reinterpret_cast<cudaStream_t>(stream)) ==
+                   cudaSuccess
+               ? CADKV_OK
+               : CADKV_ERR_CUDA;
+}
+
+int prefill_attention_status(const void *workspace, cadkv_stream_t stream)
 {
     return read_status(workspace, reinterpret_cast<cudaStream_t>(stream));
 }

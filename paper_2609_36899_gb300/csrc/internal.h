@@ -86,6 +86,25 @@ cudaError_t launch_attention(const AttnParams &p, const CUtensorMap &kmap,
                              cudaStream_t stream);
 size_t attention_smem_bytes(int head_dim);
 
+// ---------------------------------------------------------------- prefill
+
+struct PrefillParams {
+    const long long *q_offsets;  // device [batch + 1]
+    const int *context_lens;
+    const int *block_table;
+    __nv_bfloat16 *out;          // [T][Hq][D]
+    float *lse;                  // [T][Hq], nullable
+    WorkspaceHeader *hdr;
+    long long *item_prefix;      // [batch + 1]
+    long long total_q;           // rows of q / out; offsets beyond it are rejected
+    int batch, num_q_heads, num_kv_heads, group, max_pages, num_pages;
+    float scale_log2;
+};
+
+size_t prefill_smem_bytes();
+cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, const CUtensorMap &kmap,
+                           const CUtensorMap &vmap, int grid, cudaStream_t stream);
+
 // ---------------------------------------------------------------- staging
 
 struct StageParams {

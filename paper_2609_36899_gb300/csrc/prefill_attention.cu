@@ -1,0 +1,535 @@
+// prefill_attention.cu -- chunked (re-)prefill attention over the paged KV pool
+// on the 5th-generation tensor cores (tcgen05, accumulators in TMEM).
+//
+// When prepared KV state cannot be used, the destination recomputes the
+// prefix (Sec. 4.4, the fallback of late-bound KV preparation): each
+// trajectory's last C_b tokens attend causally over its paged KV.  Unlike the
+// decode step this is a dense contraction (128 query rows share every key
+// tile), so it runs on tcgen05.mma:
+//
+//  * One CTA per work item (trajectory b, KV head g, tile of 128 query rows).
+//    A row is a (query token, query head of group g) pair, token-major, so
+//    the G heads sharing a KV head share every K/V tile (GQA).
+//  * Warp 0 (TMA producer) loads the Q tile once (3-D tensor map, two 64-
+//    column panels, 128-byte swizzle) and streams K and V tiles of 128 keys
+//    (8 pages, two 2 KB boxes per page and operand) into 2-stage rings.
+//  * Warp 1 (MMA issuer, one lane) computes S_j = Q K_j^T into one of two TMEM
+//    buffers (128 lanes x 128 fp32 columns) while the softmax warps work on
+//    the other, then O += P_j V_j into a third TMEM region (V as an MN-major
+//    operand straight from the swizzled stage).
+//  * Warps 2-5 (softmax, one query row per thread = one TMEM lane) read S_j
+//    with tcgen05.ld, apply the causal mask, keep a running max (rescaling the
+//    O row in TMEM only when the max grows by more than 2^8), write P_j as
+//    bf16 into a swizzled shared-memory tile (the A operand of the PV MMA),
+//    and finally normalise O and write out and lse.
+//  * All waits are bounded; on timeout the kernel records CADKV_ERR_TIMEOUT,
+//    waits for its own copies and MMAs, frees TMEM and returns.
+#include <cfloat>
+#include <cmath>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace cadkv {
+
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr int kRows = 128;            // query rows per tile = MMA M
+constexpr int kKeys = 128;            // keys per tile = MMA N of QK^T, K of PV
+constexpr int kD = 128;               // head_dim
+constexpr int kPanel = 16384;         // 128 rows x 128 B (one 64-column panel)
+constexpr int kTileBytes = 2 * kPanel;  // 128 rows x 128 columns bf16
+constexpr int kPrefillThreads = 192;  // producer, MMA, 4 softmax warps
+constexpr float kRescaleThreshold = 8.0f;  // log2 units
+
+struct PrefillSmem {
+    uint8_t q[kTileBytes];
+    uint8_t p[kTileBytes];
+    uint8_t k[2][kTileBytes];
+    uint8_t v[2][kTileBytes];
+    uint64_t q_full, s_full[2], p_full, o_done, k_full[2], k_empty[2], v_full[2], v_empty[2],
+        mma_done;
+    uint32_t tmem_base;
+    int abort;
+};
+
+__device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo)
+{
+    uint64_t d = (uint64_t)((saddr & 0x3FFFF) >> 4);
+    d |= (uint64_t)((lbo >> 4) & 0x3FFF) << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFF) << 32;
+    d |= (uint64_t)1 << 46;  // fixed 0b001
+    d |= (uint64_t)2 << 61;  // 128-byte swizzle
+    return d;
+}
+
+// kind::f16 instruction descriptor: bf16 A/B, fp32 D, M x N, operand majors.
+__device__ __forceinline__ uint32_t idesc_bf16(int m, int n, int a_mn, int b_mn)
+{
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)a_mn << 15) |
+           ((uint32_t)b_mn << 16) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                     uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void umma_commit(uint64_t *bar)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                     smem_addr(bar))
+                 : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+#define CADKV_TMEM_LD32(taddr, r)                                                                   \
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,"   \
+                 "%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,"  \
+                 "%31}, [%32];"                                                                   \
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),          \
+                   "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]),        \
+                   "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]),    \
+                   "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),    \
+                   "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]),    \
+                   "=r"(r[30]), "=r"(r[31])                                                       \
+                 : "r"(taddr))
+
+#define CADKV_TMEM_ST32(taddr, r)                                                                   \
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,"    \
+                 "%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,"  \
+                 "%30,%31,%32};" ::"r"(taddr),                                                    \
+                 "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]),       \
+                 "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]),   \
+                 "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]),            \
+                 "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]),            \
+                 "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])             \
+                 : "memory")
+
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// ------------------------------------------------------------------ planner
+
+__global__ void __launch_bounds__(1024, 1) prefill_plan_kernel(const PrefillParams p)
+{
+    __shared__ long long warp_sums[32];
+    __shared__ long long carry_s;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int rows_per_token = p.group;
+    if (tid == 0) {
+        p.hdr->status = 0;
+        carry_s = 0;
+    }
+    __syncthreads();
+    for (int base = 0; base < p.batch; base += 1024) {
+        const int b = base + tid;
+        long long items = 0;
+        if (b < p.batch) {
+            const long long qa = p.q_offsets[b], qb = p.q_offsets[b + 1];
+            const long long c = qb - qa;
+            const int n = p.context_lens[b];
+            if (qa < 0 || qb > p.total_q || c < 0 || n < 0 || c > n ||
+                n > p.max_pages * kPageSize) {
+                record_status(&p.hdr->status, CADKV_ERR_SHAPE);
+            } else {
+                items = (long long)p.num_kv_heads * ((c * rows_per_token + kRows - 1) / kRows);
+            }
+        }
+        long long v = items;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const long long u = __shfl_up_sync(kFull, v, o);
+            if (lane >= o)
+                v += u;
+        }
+        if (lane == 31)
+            warp_sums[warp] = v;
+        __syncthreads();
+        if (warp == 0) {
+            long long w = warp_sums[lane];
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const long long u = __shfl_up_sync(kFull, w, o);
+                if (lane >= o)
+                    w += u;
+            }
+            warp_sums[lane] = w;
+        }
+        __syncthreads();
+        const long long incl = carry_s + v + (warp > 0 ? warp_sums[warp - 1] : 0);
+        if (b < p.batch)
+            p.item_prefix[b] = incl - items;
+        __syncthreads();
+        if (tid == 1023)
+            carry_s = incl;
+        __syncthreads();
+    }
+    if (tid == 0) {
+        p.item_prefix[p.batch] = carry_s;
+        p.hdr->total_work = carry_s;
+    }
+}
+
+// ------------------------------------------------------------------ attention
+
+__global__ void __launch_bounds__(kPrefillThreads, 1)
+    prefill_attention_kernel(const PrefillParams p, const __grid_constant__ CUtensorMap qmap,
+                             const __grid_constant__ CUtensorMap kmap,
+                             const __grid_constant__ CUtensorMap vmap)
+{
+    extern __shared__ uint8_t smem_raw[];
+    PrefillSmem &sm = *reinterpret_cast<PrefillSmem *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const long long total = p.hdr->total_work;
+    const long long item = blockIdx.x;
+    if (item >= total)
+        return;  // uniform across the CTA, before any barrier or TMEM use
+
+    // ---- decode the work item: (trajectory b, KV head g, query tile qt)
+    int lo = 0, hi = p.batch - 1;
+    while (lo < hi) {  // largest b with item_prefix[b] <= item
+        const int mid = (lo + hi + 1) >> 1;
+        if (p.item_prefix[mid] <= item)
+            lo = mid;
+        else
+            hi = mid - 1;
+    }
+    const int b = lo;
+    const int G = p.group;
+    const int tokens_per_tile = kRows / G;
+    const long long q0 = p.q_offsets[b];
+    const int chunk = (int)(p.q_offsets[b + 1] - q0);
+    const int n = p.context_lens[b];
+    const int qtiles = (chunk * G + kRows - 1) / kRows;
+    const int local = (int)(item - p.item_prefix[b]);
+    const int g = local / qtiles;
+    const int qt = qtiles - 1 - local % qtiles;  // heaviest tiles first
+    const int i0 = qt * tokens_per_tile;
+    const int valid_tokens = min(tokens_per_tile, chunk - i0);
+    const int chunk_start = n - chunk;
+    const int pos_max = chunk_start + i0 + valid_tokens - 1;
+    const int num_kt = (pos_max + 1 + kKeys - 1) / kKeys;
+    const int last_page = pos_max / kPageSize;  // inclusive
+
+    if (tid == 0) {
+        mbar_init(&sm.q_full, 1);
+        mbar_init(&sm.s_full[0], 1);
+        mbar_init(&sm.s_full[1], 1);
+        mbar_init(&sm.p_full, 128);
+        mbar_init(&sm.o_done, 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&sm.k_full[s], 1);
+            mbar_init(&sm.k_empty[s], 1);
+            mbar_init(&sm.v_full[s], 1);
+            mbar_init(&sm.v_empty[s], 1);
+        }
+        mbar_init(&sm.mma_done, 1);
+        sm.abort = 0;
+        fence_mbarrier_init();
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
+                         smem_addr(&sm.tmem_base))
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sm.tmem_base;
+    const uint32_t tmem_s[2] = {tmem, tmem + 128};
+    const uint32_t tmem_o = tmem + 256;
+    volatile int *abort_flag = &sm.abort;
+
+    if (warp == 0) {
+        // ============================ TMA producer ============================
+        bool ok = true;
+        int issued_k = 0, issued_v = 0;
+        if (lane == 0) {
+            prefetch_tensor_map(&qmap);
+            prefetch_tensor_map(&kmap);
+            prefetch_tensor_map(&vmap);
+            mbar_arrive_expect_tx(&sm.q_full, kTileBytes);
+            const int qy = (int)(q0 + i0);
+            for (int h = 0; h < 2; ++h)
+                tma_load_3d(sm.q + h * kPanel, &qmap, h * 64, g * G, qy, &sm.q_full);
+            const uint64_t policy = l2_evict_first_policy();
+            for (int j = 0; j < num_kt && ok; ++j) {
+                const int s = j & 1;
+                const int first_page = j * (kKeys / kPageSize);
+                const int pages = min(kKeys / kPageSize, last_page + 1 - first_page);
+                const uint32_t bytes = (uint32_t)pages * 2 * 2048;
+                for (int op = 0; op < 2 && ok; ++op) {  // K then V
+                    uint64_t *empty = op == 0 ? &sm.k_empty[s] : &sm.v_empty[s];
+                    uint64_t *full = op == 0 ? &sm.k_full[s] : &sm.v_full[s];
+                    uint8_t *dst = op == 0 ? sm.k[s] : sm.v[s];
+                    const CUtensorMap *map = op == 0 ? &kmap : &vmap;
+                    if (j >= 2)
+                        ok = mbar_wait(empty, ((j >> 1) + 1) & 1, abort_flag);
+                    if (!ok)
+                        break;
+                    mbar_arrive_expect_tx(full, bytes);
+                    for (int pg = 0; pg < pages; ++pg) {
+                        int phys = p.block_table[(size_t)b * p.max_pages + first_page + pg];
+                        if (phys < 0 || phys >= p.num_pages) {
+                            record_status(&p.hdr->status, CADKV_ERR_OOB);
+                            phys = 0;
+                        }
+                        const int y = (phys * p.num_kv_heads + g) * kPageSize;
+                        tma_load_2d(dst + pg * 2048, map, 0, y, full, policy);
+                        tma_load_2d(dst + kPanel + pg * 2048, map, 64, y, full, policy);
+                    }
+                    if (op == 0)
+                        ++issued_k;
+                    else
+                        ++issued_v;
+                }
+            }
+            if (!ok) {
+                *abort_flag = 1;
+                record_status(&p.hdr->status, CADKV_ERR_TIMEOUT);
+            }
+            // every copy this warp started must land before the CTA exits
+            volatile int never = 0;
+            mbar_wait(&sm.q_full, 0, &never);
+            for (int j = max(0, issued_k - 2); j < issued_k; ++j)
+                mbar_wait(&sm.k_full[j & 1], (j >> 1) & 1, &never);
+            for (int j = max(0, issued_v - 2); j < issued_v; ++j)
+                mbar_wait(&sm.v_full[j & 1], (j >> 1) & 1, &never);
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ============================ MMA issuer ============================
+        if (lane == 0) {
+            const uint32_t id_qk = idesc_bf16(kRows, kKeys, 0, 0);
+            const uint32_t id_pv = idesc_bf16(kRows, kD, 0, 1);
+            bool ok = mbar_wait(&sm.q_full, 0, abort_flag) && mbar_wait(&sm.k_full[0], 0, abort_flag);
+            auto issue_qk = [&](int j) {
+                const int s = j & 1;
+                tc_fence_after();
+#pragma unroll
+                for (int k = 0; k < kD / 16; ++k) {
+                    const int atom = k >> 2, kin = k & 3;
+                    const uint64_t a = desc_sw128(smem_addr(sm.q + atom * kPanel) + kin * 32, 16, 1024);
+                    const uint64_t bd = desc_sw128(smem_addr(sm.k[s] + atom * kPanel) + kin * 32, 16, 1024);
+                    umma(tmem_s[s], a, bd, id_qk, k > 0);
+                }
+                umma_commit(&sm.s_full[s]);
+            };
+            if (ok)
+                issue_qk(0);
+            for (int j = 0; j < num_kt && ok; ++j) {
+                const int s = j & 1;
+                if (j + 1 < num_kt) {
+                    ok = mbar_wait(&sm.k_full[(j + 1) & 1], ((j + 1) >> 1) & 1, abort_flag);
+                    if (!ok)
+                        break;
+                    issue_qk(j + 1);  // S buffer (j+1)&1 was released with P_{j-1}
+                }
+                ok = mbar_wait(&sm.p_full, j & 1, abort_flag) &&
+                     mbar_wait(&sm.v_full[s], (j >> 1) & 1, abort_flag);
+                if (!ok)
+                    break;
+                tc_fence_after();
+#pragma unroll
+                for (int k = 0; k < kKeys / 16; ++k) {
+                    const int atom = k >> 2, kin = k & 3;
+                    const uint64_t a = desc_sw128(smem_addr(sm.p + atom * kPanel) + kin * 32, 16, 1024);
+                    const uint64_t bd = desc_sw128(smem_addr(sm.v[s]) + k * 2048, kPanel, 1024);
+                    umma(tmem_o, a, bd, id_pv, (j > 0 || k > 0) ? 1u : 0u);
+                }
+                umma_commit(&sm.o_done);
+                umma_commit(&sm.k_empty[s]);
+                umma_commit(&sm.v_empty[s]);
+            }
+            if (!ok) {
+                *abort_flag = 1;
+                record_status(&p.hdr->status, CADKV_ERR_TIMEOUT);
+            }
+            // all MMAs this thread issued complete before TMEM is freed
+            umma_commit(&sm.mma_done);
+            volatile int never = 0;
+            mbar_wait(&sm.mma_done, 0, &never);
+        }
+        __syncwarp();
+    } else {
+        // ============================ softmax warps ============================
+        const int row = 32 * (warp & 3) + lane;  // TMEM lane = query row
+        const uint32_t lane_base = (uint32_t)(32 * (warp & 3)) << 16;
+        const int token = row / G, head = row % G;
+        const bool row_valid = token < valid_tokens;
+        const int pos_row = row_valid ? chunk_start + i0 + token : pos_max;
+        const float scale = p.scale_log2;
+        float m = -INFINITY, l = 0.f;
+        bool ok = true;
+        uint8_t *prow = sm.p + row * 128;
+        for (int j = 0; j < num_kt && ok; ++j) {
+            const int s = j & 1;
+            ok = __all_sync(kFull, mbar_wait(&sm.s_full[s], (j >> 1) & 1, abort_flag));
+            if (!ok)
+                break;
+            tc_fence_after();
+            const int key0 = j * kKeys;
+            // pass 1: masked row max
+            float mx = -INFINITY;
+            for (int c = 0; c < 4; ++c) {
+                uint32_t r[32];
+                CADKV_TMEM_LD32(tmem_s[s] + lane_base + c * 32, r);
+                tmem_wait_ld();
+#pragma unroll
+                for (int e = 0; e < 32; ++e)
+                    if (key0 + c * 32 + e <= pos_row)
+                        mx = fmaxf(mx, __uint_as_float(r[e]) * scale);
+            }
+            const float m_new = fmaxf(m, mx);
+            // P smem and O are free once the previous PV has completed
+            if (j > 0) {
+                ok = __all_sync(kFull, mbar_wait(&sm.o_done, (j - 1) & 1, abort_flag));
+                if (!ok)
+                    break;
+                tc_fence_after();
+            }
+            // tcgen05.ld/st are warp-collective: the whole warp rescales when any
+            // lane's max grew past the threshold (rescaling to the true max is
+            // always correct, only skipping it needs the bound).
+            if (__any_sync(kFull, m_new > m + kRescaleThreshold)) {
+                const float alpha = exp2_approx(m - m_new);  // 0 on the first tile
+                if (j > 0) {
+                    for (int c = 0; c < 4; ++c) {
+                        uint32_t r[32];
+                        CADKV_TMEM_LD32(tmem_o + lane_base + c * 32, r);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 32; ++e)
+                            r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+                        CADKV_TMEM_ST32(tmem_o + lane_base + c * 32, r);
+                    }
+                    tmem_wait_st();
+                }
+                l *= alpha;
+                m = m_new;
+            }
+            // pass 2: P = 2^(s - m) as bf16 into the swizzled A tile
+            for (int c = 0; c < 4; ++c) {
+                uint32_t r[32];
+                CADKV_TMEM_LD32(tmem_s[s] + lane_base + c * 32, r);
+                tmem_wait_ld();
+                uint32_t packed[16];
+#pragma unroll
+                for (int e = 0; e < 32; e += 2) {
+                    const int key = key0 + c * 32 + e;
+                    const float p0 = key <= pos_row ? exp2_approx(__uint_as_float(r[e]) * scale - m) : 0.f;
+                    const float p1 = key + 1 <= pos_row ? exp2_approx(__uint_as_float(r[e + 1]) * scale - m) : 0.f;
+                    l += p0 + p1;
+                    packed[e >> 1] = pack_bf16x2(p0, p1);
+                }
+                // keys c*32 .. c*32+31 = 16-byte chunks 4c .. 4c+3 of the row
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    const int chunk16 = c * 4 + q4;           // 0..15 across both panels
+                    const int panel = chunk16 >> 3, cin = chunk16 & 7;
+                    uint4 *dst = reinterpret_cast<uint4 *>(prow + panel * kPanel + ((cin ^ (row & 7)) << 4));
+                    *dst = make_uint4(packed[4 * q4], packed[4 * q4 + 1], packed[4 * q4 + 2], packed[4 * q4 + 3]);
+                }
+            }
+            if (j == num_kt - 1) {
+                // Zero V rows past pos_max: those keys may hold NaN (slots past n_b,
+                // or pages never loaded) and 0 * NaN would poison the PV sum.
+                ok = __all_sync(kFull, mbar_wait(&sm.v_full[s], (j >> 1) & 1, abort_flag));
+                if (!ok)
+                    break;
+                const int key_row = tid - 64;              // 0..127
+                if (key0 + key_row > pos_max) {
+                    uint4 *r0 = reinterpret_cast<uint4 *>(sm.v[s] + key_row * 128);
+                    uint4 *r1 = reinterpret_cast<uint4 *>(sm.v[s] + kPanel + key_row * 128);
+#pragma unroll
+                    for (int c16 = 0; c16 < 8; ++c16) {
+                        r0[c16] = make_uint4(0, 0, 0, 0);
+                        r1[c16] = make_uint4(0, 0, 0, 0);
+                    }
+                }
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            mbar_arrive(&sm.p_full);
+        }
+        // ---- epilogue: O / l -> out, lse
+        if (ok) {
+            ok = __all_sync(kFull, mbar_wait(&sm.o_done, (num_kt - 1) & 1, abort_flag));
+            tc_fence_after();
+        }
+        if (ok) {
+            const float inv = 1.f / l;
+            __nv_bfloat16 *orow = p.out + ((size_t)(q0 + i0 + token) * p.num_q_heads + g * G + head) * kD;
+            for (int c = 0; c < 4; ++c) {
+                uint32_t r[32];
+                CADKV_TMEM_LD32(tmem_o + lane_base + c * 32, r);
+                tmem_wait_ld();
+                if (row_valid) {
+                    uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) {
+                        uint4 v;
+                        v.x = pack_bf16x2(__uint_as_float(r[8 * q4 + 0]) * inv, __uint_as_float(r[8 * q4 + 1]) * inv);
+                        v.y = pack_bf16x2(__uint_as_float(r[8 * q4 + 2]) * inv, __uint_as_float(r[8 * q4 + 3]) * inv);
+                        v.z = pack_bf16x2(__uint_as_float(r[8 * q4 + 4]) * inv, __uint_as_float(r[8 * q4 + 5]) * inv);
+                        v.w = pack_bf16x2(__uint_as_float(r[8 * q4 + 6]) * inv, __uint_as_float(r[8 * q4 + 7]) * inv);
+                        dst[q4] = v;
+                    }
+                }
+            }
+            if (row_valid && p.lse)
+                p.lse[(size_t)(q0 + i0 + token) * p.num_q_heads + g * G + head] =
+                    (m + __log2f(l)) * kLn2;
+        }
+        if (!ok && lane == 0) {
+            *abort_flag = 1;
+            record_status(&p.hdr->status, CADKV_ERR_TIMEOUT);
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem) : "memory");
+    }
+}
+
+}  // namespace
+
+size_t prefill_smem_bytes() { return sizeof(PrefillSmem) + 1024; }
+
+cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, const CUtensorMap &kmap,
+                           const CUtensorMap &vmap, int grid, cudaStream_t stream)
+{
+    static bool configured = false;
+    const size_t smem = prefill_smem_bytes();
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(prefill_attention_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess)
+            return e;
+        configured = true;
+    }
+    prefill_plan_kernel<<<1, 1024, 0, stream>>>(p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess || grid == 0)
+        return e;
+    prefill_attention_kernel<<<grid, kPrefillThreads, smem, stream>>>(p, qmap, kmap, vmap);
+    return cudaGetLastError();
+}
+
+}  // namespace cadkv

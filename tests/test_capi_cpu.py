@@ -104,3 +104,23 @@ def test_read_probe_rejects_on_host(lib):
     assert lib.cadkv_hbm_read_probe(P((1 << 12) + 4), 16, P(1 << 12), None) == \
         STATUS["CADKV_ERR_INVALID"]
     assert lib.cadkv_hbm_read_probe(P(1 << 12), 0, P(1 << 12), None) == 0
+
+
+def test_prefill_rejects_on_host(lib):
+    P = ctypes.c_void_p
+    a = P(1 << 12)
+
+    def call(**over):
+        args = dict(q=a, offs=a, k=a, v=a, bt=a, cl=a, out=a, batch=2, total=8, hq=8, hkv=2,
+                    d=128, page=16, num_pages=4, max_pages=4)
+        args.update(over)
+        return lib.prefill_attention(args["q"], args["offs"], args["k"], args["v"], args["bt"],
+                                     args["cl"], args["out"], None, args["batch"], args["total"],
+                                     args["hq"], args["hkv"], args["d"], args["page"],
+                                     args["num_pages"], args["max_pages"], a, 1 << 20, None)
+    assert call(d=64) == STATUS["CADKV_ERR_UNSUPPORTED"]
+    assert call(hq=6, hkv=2) == STATUS["CADKV_ERR_UNSUPPORTED"]      # G = 3
+    assert call(hq=6, hkv=4) == STATUS["CADKV_ERR_SHAPE"]
+    assert call(q=None) == STATUS["CADKV_ERR_INVALID"]
+    assert call(offs=P((1 << 12) + 4)) == STATUS["CADKV_ERR_INVALID"]
+    assert call(total=0) == 0

@@ -1,0 +1,98 @@
+"""GPU chunked prefill attention (tcgen05 kernel, through the C ABI) against
+the fp64 oracle on the same bf16 inputs, within the decode tolerances."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2609_36899_gb300 as cadkv
+from paper_2609_36899_gb300 import STATUS
+from paper_2609_36899_gb300.workloads import bf16_bits
+from _gpu_util import assert_close, make_batch
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2609_36899_gb300 import build
+    build.build()
+
+
+def _case(lens, chunks, hq, hkv, seed):
+    batch = make_batch(lens, hq, hkv, 128, seed=seed)     # NaN past n_b in the pool
+    offs = np.concatenate([[0], np.cumsum(chunks)]).astype(np.int64)
+    g = torch.Generator().manual_seed(seed + 1)
+    q = torch.randn((int(offs[-1]), hq, 128), generator=g).to(torch.bfloat16)
+    return batch, offs, q
+
+
+def _run(batch, offs, q):
+    out, lse, ws = cadkv.prefill_attention(
+        q.cuda(), torch.from_numpy(offs).cuda(), batch.k_pages.cuda(), batch.v_pages.cuda(),
+        torch.from_numpy(batch.block_table).cuda(), torch.from_numpy(batch.context_lens).cuda())
+    torch.cuda.synchronize()
+    return out, lse, ws
+
+
+def _oracle(batch, offs, q):
+    return oracle.prefill_attention(bf16_bits(q), offs, bf16_bits(batch.k_pages),
+                                    bf16_bits(batch.v_pages), batch.block_table,
+                                    batch.context_lens)
+
+
+@pytest.mark.parametrize("g", [1, 2, 4, 8])
+def test_prefill_small(g):
+    lens, chunks = [40, 300, 17, 130], [40, 5, 17, 129]
+    batch, offs, q = _case(lens, chunks, 2 * g, 2, seed=400 + g)
+    out, lse, ws = _run(batch, offs, q)
+    assert cadkv.prefill_attention_status(ws) == 0
+    ref, ref_lse = _oracle(batch, offs, q)
+    assert_close(out, lse, ref, ref_lse, f"prefill G={g}")
+
+
+def test_prefill_many_tiles():
+    """Chunks spanning several query tiles and key tiles, ragged everywhere."""
+    lens, chunks = [1000, 700, 257], [300, 1, 257]
+    batch, offs, q = _case(lens, chunks, 8, 2, seed=410)
+    out, lse, ws = _run(batch, offs, q)
+    ref, ref_lse = _oracle(batch, offs, q)
+    assert_close(out, lse, ref, ref_lse, "prefill many tiles")
+
+
+def test_prefill_qwen_shape():
+    """32 query / 8 KV heads (G = 4), contexts of a few thousand tokens."""
+    lens, chunks = [3000, 4500], [256, 130]
+    batch, offs, q = _case(lens, chunks, 32, 8, seed=420)
+    out, lse, ws = _run(batch, offs, q)
+    ref, ref_lse = _oracle(batch, offs, q)
+    assert_close(out, lse, ref, ref_lse, "prefill 32/8")
+
+
+def test_prefill_chunk_of_one_matches_decode():
+    lens = [77, 1, 513]
+    batch, offs, q = _case(lens, [1, 1, 1], 16, 2, seed=430)
+    out, lse, _ = _run(batch, offs, q)
+    dq = q.view(3, 16, 128).cuda()
+    dec_out, dec_lse = cadkv.decode_attention(
+        dq, batch.k_pages.cuda(), batch.v_pages.cuda(),
+        torch.from_numpy(batch.block_table).cuda(), torch.from_numpy(batch.context_lens).cuda())
+    ref, ref_lse = _oracle(batch, offs, q)
+    assert_close(out, lse, ref, ref_lse, "prefill C=1")
+    assert_close(dec_out, dec_lse, ref.reshape(3, 16, 128), ref_lse.reshape(3, 16), "decode")
+
+
+def test_prefill_rejects_chunk_longer_than_context():
+    batch, offs, q = _case([20, 40], [5, 10], 4, 1, seed=440)
+    cl = torch.from_numpy(batch.context_lens).cuda()
+    cl[1] = 7                      # chunk of 10 cannot end at position 6
+    out = torch.full((15, 4, 128), 3.0, dtype=torch.bfloat16, device="cuda")
+    _, _, ws = cadkv.prefill_attention(
+        q.cuda(), torch.from_numpy(offs).cuda(), batch.k_pages.cuda(), batch.v_pages.cuda(),
+        torch.from_numpy(batch.block_table).cuda(), cl, out=out)
+    assert cadkv.prefill_attention_status(ws) == STATUS["CADKV_ERR_SHAPE"]
+    assert torch.all(out[5:] == 3.0)                     # trajectory 1 untouched
+    ref, ref_lse = oracle.prefill_attention(
+        bf16_bits(q[:5]), offs[:2], bf16_bits(batch.k_pages), bf16_bits(batch.v_pages),
+        batch.block_table[:1], batch.context_lens[:1])
+    assert_close(out[:5], None, ref, ref_lse, "trajectory 0")
