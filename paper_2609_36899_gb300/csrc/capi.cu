@@ -593,7 +593,7 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return CADKV_ERR_CUDA;
     }
-    int whole = 0;
+    int whole = 0;  // the prefill kernel uses 2-D boxes of one 64-column panel
     if (encode_pages_map(&kmap, k_pages, num_pages, num_kv_heads, head_dim, false, &whole) !=
             CADKV_OK ||
         encode_pages_map(&vmap, v_pages, num_pages, num_kv_heads, head_dim, false, &whole) !=

@@ -12,14 +12,17 @@
 //    the G heads sharing a KV head share every K/V tile (GQA).
 //  * Warp 0 (TMA producer) loads the Q tile once (3-D tensor map, two 64-
 //    column panels, 128-byte swizzle) and streams K and V tiles of 128 keys
-//    (8 pages, two 2 KB boxes per page and operand) into 2-stage rings.
+//    (8 pages, two 2 KB boxes per page and operand, issued from 32 lanes at
+//    once) into 2-stage rings.
 //  * Warp 1 (MMA issuer, one lane) computes S_j = Q K_j^T into one of two TMEM
 //    buffers (128 lanes x 128 fp32 columns) while the softmax warps work on
 //    the other, then O += P_j V_j into a third TMEM region (V as an MN-major
 //    operand straight from the swizzled stage).
-//  * Warps 2-5 (softmax, one query row per thread = one TMEM lane) read S_j
-//    with tcgen05.ld, apply the causal mask, keep a running max (rescaling the
-//    O row in TMEM only when the max grows by more than 2^8), write P_j as
+//  * Warps 2-9 (softmax, two warpgroups; a thread owns one query row = one
+//    TMEM lane and 64 of its 128 key columns) read S_j with tcgen05.ld, apply
+//    the causal mask (only on tiles that cross the diagonal), combine the two
+//    halves' row maxima through shared memory, keep a running max (rescaling
+//    the O row in TMEM only when the max grows by more than 2^8), write P_j as
 //    bf16 into a swizzled shared-memory tile (the A operand of the PV MMA),
 //    and finally normalise O and write out and lse.
 //  * All waits are bounded; on timeout the kernel records CADKV_ERR_TIMEOUT,
@@ -41,7 +44,9 @@ constexpr int kKeys = 128;            // keys per tile = MMA N of QK^T, K of PV
 constexpr int kD = 128;               // head_dim
 constexpr int kPanel = 16384;         // 128 rows x 128 B (one 64-column panel)
 constexpr int kTileBytes = 2 * kPanel;  // 128 rows x 128 columns bf16
-constexpr int kPrefillThreads = 192;  // producer, MMA, 4 softmax warps
+constexpr int kPageBlock = kPageSize * kD * 2;  // one (page, head) block: 4 KB
+constexpr int kSoftmaxThreads = 256;  // two warpgroups, 64 key columns of every row each
+constexpr int kPrefillThreads = 64 + kSoftmaxThreads;  // producer, MMA, softmax
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 struct PrefillSmem {
@@ -49,8 +54,9 @@ struct PrefillSmem {
     uint8_t p[kTileBytes];
     uint8_t k[2][kTileBytes];
     uint8_t v[2][kTileBytes];
+    float red[2][2][kRows];  // [tile parity][half][row]: partial row maxima (sums at the end)
     uint64_t q_full, s_full[2], p_full, o_done, k_full[2], k_empty[2], v_full[2], v_empty[2],
-        mma_done;
+        mma_done, pair;
     uint32_t tmem_base;
     int abort;
 };
@@ -227,7 +233,8 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
         mbar_init(&sm.q_full, 1);
         mbar_init(&sm.s_full[0], 1);
         mbar_init(&sm.s_full[1], 1);
-        mbar_init(&sm.p_full, 128);
+        mbar_init(&sm.p_full, kSoftmaxThreads);
+        mbar_init(&sm.pair, kSoftmaxThreads);
         mbar_init(&sm.o_done, 1);
         for (int s = 0; s < 2; ++s) {
             mbar_init(&sm.k_full[s], 1);
@@ -255,8 +262,15 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
 
     if (warp == 0) {
         // ============================ TMA producer ============================
+        // Q: one 3-D tensor-map load (two 64-column panels).  K, V: a tile's 8
+        // pages as 2 KB boxes (16 tokens x one 64-column panel) landing in the
+        // panel layout the MMAs read (row = key).  Lane 0 waits for free stages
+        // and arms the barriers; then all 32 lanes issue one box each (lanes
+        // 0-15: K, 16-31: V; page = (lane/2)%8, panel = lane%2) so a tile's 32
+        // copies start together.
         bool ok = true;
-        int issued_k = 0, issued_v = 0;
+        int issued = 0;
+        const uint64_t policy = l2_evict_first_policy();
         if (lane == 0) {
             prefetch_tensor_map(&qmap);
             prefetch_tensor_map(&kmap);
@@ -265,38 +279,38 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             const int qy = (int)(q0 + i0);
             for (int h = 0; h < 2; ++h)
                 tma_load_3d(sm.q + h * kPanel, &qmap, h * 64, g * G, qy, &sm.q_full);
-            const uint64_t policy = l2_evict_first_policy();
-            for (int j = 0; j < num_kt && ok; ++j) {
-                const int s = j & 1;
-                const int first_page = j * (kKeys / kPageSize);
-                const int pages = min(kKeys / kPageSize, last_page + 1 - first_page);
-                const uint32_t bytes = (uint32_t)pages * 2 * 2048;
-                for (int op = 0; op < 2 && ok; ++op) {  // K then V
-                    uint64_t *empty = op == 0 ? &sm.k_empty[s] : &sm.v_empty[s];
-                    uint64_t *full = op == 0 ? &sm.k_full[s] : &sm.v_full[s];
-                    uint8_t *dst = op == 0 ? sm.k[s] : sm.v[s];
-                    const CUtensorMap *map = op == 0 ? &kmap : &vmap;
-                    if (j >= 2)
-                        ok = mbar_wait(empty, ((j >> 1) + 1) & 1, abort_flag);
-                    if (!ok)
-                        break;
-                    mbar_arrive_expect_tx(full, bytes);
-                    for (int pg = 0; pg < pages; ++pg) {
-                        int phys = p.block_table[(size_t)b * p.max_pages + first_page + pg];
-                        if (phys < 0 || phys >= p.num_pages) {
-                            record_status(&p.hdr->status, CADKV_ERR_OOB);
-                            phys = 0;
-                        }
-                        const int y = (phys * p.num_kv_heads + g) * kPageSize;
-                        tma_load_2d(dst + pg * 2048, map, 0, y, full, policy);
-                        tma_load_2d(dst + kPanel + pg * 2048, map, 64, y, full, policy);
-                    }
-                    if (op == 0)
-                        ++issued_k;
-                    else
-                        ++issued_v;
+        }
+        const int op = lane >> 4, pg = (lane >> 1) & 7, hh = lane & 1;
+        for (int j = 0; j < num_kt; ++j) {
+            const int s = j & 1;
+            const int first_page = j * (kKeys / kPageSize);
+            const int pages = min(kKeys / kPageSize, last_page + 1 - first_page);
+            if (lane == 0) {
+                if (j >= 2)
+                    ok = mbar_wait(&sm.k_empty[s], ((j >> 1) + 1) & 1, abort_flag) &&
+                         mbar_wait(&sm.v_empty[s], ((j >> 1) + 1) & 1, abort_flag);
+                if (ok) {
+                    mbar_arrive_expect_tx(&sm.k_full[s], (uint32_t)pages * kPageBlock);
+                    mbar_arrive_expect_tx(&sm.v_full[s], (uint32_t)pages * kPageBlock);
                 }
             }
+            ok = __shfl_sync(kFull, ok ? 1 : 0, 0) != 0;
+            if (!ok)
+                break;
+            if (pg < pages) {
+                int phys = p.block_table[(size_t)b * p.max_pages + first_page + pg];
+                if (phys < 0 || phys >= p.num_pages) {
+                    record_status(&p.hdr->status, CADKV_ERR_OOB);
+                    phys = 0;
+                }
+                const int y = (phys * p.num_kv_heads + g) * kPageSize;
+                uint8_t *dst = (op == 0 ? sm.k[s] : sm.v[s]) + hh * kPanel + pg * 2048;
+                tma_load_2d(dst, op == 0 ? &kmap : &vmap, hh * 64, y,
+                            op == 0 ? &sm.k_full[s] : &sm.v_full[s], policy);
+            }
+            ++issued;
+        }
+        if (lane == 0) {
             if (!ok) {
                 *abort_flag = 1;
                 record_status(&p.hdr->status, CADKV_ERR_TIMEOUT);
@@ -304,10 +318,10 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             // every copy this warp started must land before the CTA exits
             volatile int never = 0;
             mbar_wait(&sm.q_full, 0, &never);
-            for (int j = max(0, issued_k - 2); j < issued_k; ++j)
+            for (int j = max(0, issued - 2); j < issued; ++j) {
                 mbar_wait(&sm.k_full[j & 1], (j >> 1) & 1, &never);
-            for (int j = max(0, issued_v - 2); j < issued_v; ++j)
                 mbar_wait(&sm.v_full[j & 1], (j >> 1) & 1, &never);
+            }
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -327,6 +341,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                     umma(tmem_s[s], a, bd, id_qk, k > 0);
                 }
                 umma_commit(&sm.s_full[s]);
+                umma_commit(&sm.k_empty[s]);  // K_j is read only by S_j: free it early
             };
             if (ok)
                 issue_qk(0);
@@ -343,6 +358,8 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                 if (!ok)
                     break;
                 tc_fence_after();
+                // O += P V: V as an MN-major operand (64-column panels 16 KB apart,
+                // 8-key groups 1 KB apart); K step k = keys 16k .. 16k+15.
 #pragma unroll
                 for (int k = 0; k < kKeys / 16; ++k) {
                     const int atom = k >> 2, kin = k & 3;
@@ -351,7 +368,6 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                     umma(tmem_o, a, bd, id_pv, (j > 0 || k > 0) ? 1u : 0u);
                 }
                 umma_commit(&sm.o_done);
-                umma_commit(&sm.k_empty[s]);
                 umma_commit(&sm.v_empty[s]);
             }
             if (!ok) {
@@ -366,33 +382,61 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
         __syncwarp();
     } else {
         // ============================ softmax warps ============================
+        // Warp w (2..9) owns TMEM lane quarter w % 4 (rows 32*(w%4) ..) and key
+        // columns 64*half .. 64*half+63 of every tile, half = (w - 2) / 4.  The two
+        // halves of a row combine their maxima through shared memory.
+        const int half = (warp - 2) >> 2;
         const int row = 32 * (warp & 3) + lane;  // TMEM lane = query row
         const uint32_t lane_base = (uint32_t)(32 * (warp & 3)) << 16;
+        const uint32_t col0 = 64u * half;
         const int token = row / G, head = row % G;
         const bool row_valid = token < valid_tokens;
         const int pos_row = row_valid ? chunk_start + i0 + token : pos_max;
+        const int pos_min = chunk_start + i0;  // smallest position of any row in the tile
         const float scale = p.scale_log2;
         float m = -INFINITY, l = 0.f;
+        uint32_t pair_phase = 0;
         bool ok = true;
-        uint8_t *prow = sm.p + row * 128;
+        uint8_t *prow = sm.p + half * kPanel + row * 128;
+        auto pair_sync = [&]() {
+            mbar_arrive(&sm.pair);
+            const bool done = mbar_wait(&sm.pair, pair_phase, abort_flag);
+            pair_phase ^= 1u;
+            return __all_sync(kFull, done);
+        };
         for (int j = 0; j < num_kt && ok; ++j) {
             const int s = j & 1;
             ok = __all_sync(kFull, mbar_wait(&sm.s_full[s], (j >> 1) & 1, abort_flag));
             if (!ok)
                 break;
             tc_fence_after();
-            const int key0 = j * kKeys;
-            // pass 1: masked row max
+            const int key0 = j * kKeys + (int)col0;
+            // keys key0 .. key0+63 are all visible to every row of the tile?
+            const bool full_tile = key0 + 63 <= pos_min;
+            uint32_t r[64];
+            CADKV_TMEM_LD32(tmem_s[s] + lane_base + col0, r);
+            CADKV_TMEM_LD32(tmem_s[s] + lane_base + col0 + 32, (r + 32));
+            tmem_wait_ld();
+            float x[64];
             float mx = -INFINITY;
-            for (int c = 0; c < 4; ++c) {
-                uint32_t r[32];
-                CADKV_TMEM_LD32(tmem_s[s] + lane_base + c * 32, r);
-                tmem_wait_ld();
+            if (full_tile) {
 #pragma unroll
-                for (int e = 0; e < 32; ++e)
-                    if (key0 + c * 32 + e <= pos_row)
-                        mx = fmaxf(mx, __uint_as_float(r[e]) * scale);
+                for (int e = 0; e < 64; ++e) {
+                    x[e] = __uint_as_float(r[e]) * scale;
+                    mx = fmaxf(mx, x[e]);
+                }
+            } else {
+#pragma unroll
+                for (int e = 0; e < 64; ++e) {
+                    x[e] = key0 + e <= pos_row ? __uint_as_float(r[e]) * scale : -INFINITY;
+                    mx = fmaxf(mx, x[e]);
+                }
             }
+            sm.red[s][half][row] = mx;
+            ok = pair_sync();
+            if (!ok)
+                break;
+            mx = fmaxf(mx, sm.red[s][half ^ 1][row]);
             const float m_new = fmaxf(m, mx);
             // P smem and O are free once the previous PV has completed
             if (j > 0) {
@@ -403,46 +447,38 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             }
             // tcgen05.ld/st are warp-collective: the whole warp rescales when any
             // lane's max grew past the threshold (rescaling to the true max is
-            // always correct, only skipping it needs the bound).
+            // always correct, only skipping it needs the bound).  Both halves of a
+            // row see the same maxima, so they take the same decision.
             if (__any_sync(kFull, m_new > m + kRescaleThreshold)) {
                 const float alpha = exp2_approx(m - m_new);  // 0 on the first tile
                 if (j > 0) {
-                    for (int c = 0; c < 4; ++c) {
-                        uint32_t r[32];
-                        CADKV_TMEM_LD32(tmem_o + lane_base + c * 32, r);
+                    for (int c = 0; c < 2; ++c) {
+                        uint32_t o[32];
+                        CADKV_TMEM_LD32(tmem_o + lane_base + col0 + c * 32, o);
                         tmem_wait_ld();
 #pragma unroll
                         for (int e = 0; e < 32; ++e)
-                            r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-                        CADKV_TMEM_ST32(tmem_o + lane_base + c * 32, r);
+                            o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+                        CADKV_TMEM_ST32(tmem_o + lane_base + col0 + c * 32, o);
                     }
                     tmem_wait_st();
                 }
                 l *= alpha;
                 m = m_new;
             }
-            // pass 2: P = 2^(s - m) as bf16 into the swizzled A tile
-            for (int c = 0; c < 4; ++c) {
-                uint32_t r[32];
-                CADKV_TMEM_LD32(tmem_s[s] + lane_base + c * 32, r);
-                tmem_wait_ld();
-                uint32_t packed[16];
+            // P = 2^(x - m) as bf16: keys col0 .. col0+63 are panel `half` of the row
 #pragma unroll
-                for (int e = 0; e < 32; e += 2) {
-                    const int key = key0 + c * 32 + e;
-                    const float p0 = key <= pos_row ? exp2_approx(__uint_as_float(r[e]) * scale - m) : 0.f;
-                    const float p1 = key + 1 <= pos_row ? exp2_approx(__uint_as_float(r[e + 1]) * scale - m) : 0.f;
+            for (int cin = 0; cin < 8; ++cin) {
+                uint32_t packed[4];
+#pragma unroll
+                for (int e2 = 0; e2 < 4; ++e2) {
+                    const float p0 = exp2_approx(x[8 * cin + 2 * e2] - m);
+                    const float p1 = exp2_approx(x[8 * cin + 2 * e2 + 1] - m);
                     l += p0 + p1;
-                    packed[e >> 1] = pack_bf16x2(p0, p1);
+                    packed[e2] = pack_bf16x2(p0, p1);
                 }
-                // keys c*32 .. c*32+31 = 16-byte chunks 4c .. 4c+3 of the row
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    const int chunk16 = c * 4 + q4;           // 0..15 across both panels
-                    const int panel = chunk16 >> 3, cin = chunk16 & 7;
-                    uint4 *dst = reinterpret_cast<uint4 *>(prow + panel * kPanel + ((cin ^ (row & 7)) << 4));
-                    *dst = make_uint4(packed[4 * q4], packed[4 * q4 + 1], packed[4 * q4 + 2], packed[4 * q4 + 3]);
-                }
+                *reinterpret_cast<uint4 *>(prow + ((cin ^ (row & 7)) << 4)) =
+                    make_uint4(packed[0], packed[1], packed[2], packed[3]);
             }
             if (j == num_kt - 1) {
                 // Zero V rows past pos_max: those keys may hold NaN (slots past n_b,
@@ -450,47 +486,53 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                 ok = __all_sync(kFull, mbar_wait(&sm.v_full[s], (j >> 1) & 1, abort_flag));
                 if (!ok)
                     break;
-                const int key_row = tid - 64;              // 0..127
-                if (key0 + key_row > pos_max) {
-                    uint4 *r0 = reinterpret_cast<uint4 *>(sm.v[s] + key_row * 128);
-                    uint4 *r1 = reinterpret_cast<uint4 *>(sm.v[s] + kPanel + key_row * 128);
+                const int t = tid - 64;                    // 0..255
+                const int key_row = t & 127, hv = t >> 7;
+                if (j * kKeys + key_row > pos_max) {
+                    uint4 *rz = reinterpret_cast<uint4 *>(sm.v[s] + hv * kPanel + key_row * 128);
 #pragma unroll
-                    for (int c16 = 0; c16 < 8; ++c16) {
-                        r0[c16] = make_uint4(0, 0, 0, 0);
-                        r1[c16] = make_uint4(0, 0, 0, 0);
-                    }
+                    for (int c16 = 0; c16 < 8; ++c16)
+                        rz[c16] = make_uint4(0, 0, 0, 0);
                 }
             }
             fence_proxy_async_smem();
             tc_fence_before();
             mbar_arrive(&sm.p_full);
         }
-        // ---- epilogue: O / l -> out, lse
+        // ---- epilogue: combine the two halves' sums, O / l -> out, lse
         if (ok) {
+            // the last tile's maxima have been read by both halves (both passed the
+            // pair barrier of that tile), so parity slot 0/1 of the last tile is free
+            sm.red[num_kt & 1][half][row] = l;
+            ok = pair_sync();
+        }
+        if (ok) {
+            l += sm.red[num_kt & 1][half ^ 1][row];
             ok = __all_sync(kFull, mbar_wait(&sm.o_done, (num_kt - 1) & 1, abort_flag));
             tc_fence_after();
         }
         if (ok) {
             const float inv = 1.f / l;
-            __nv_bfloat16 *orow = p.out + ((size_t)(q0 + i0 + token) * p.num_q_heads + g * G + head) * kD;
-            for (int c = 0; c < 4; ++c) {
-                uint32_t r[32];
-                CADKV_TMEM_LD32(tmem_o + lane_base + c * 32, r);
+            __nv_bfloat16 *orow =
+                p.out + ((size_t)(q0 + i0 + token) * p.num_q_heads + g * G + head) * kD + col0;
+            for (int c = 0; c < 2; ++c) {
+                uint32_t o[32];
+                CADKV_TMEM_LD32(tmem_o + lane_base + col0 + c * 32, o);
                 tmem_wait_ld();
                 if (row_valid) {
                     uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
 #pragma unroll
                     for (int q4 = 0; q4 < 4; ++q4) {
                         uint4 v;
-                        v.x = pack_bf16x2(__uint_as_float(r[8 * q4 + 0]) * inv, __uint_as_float(r[8 * q4 + 1]) * inv);
-                        v.y = pack_bf16x2(__uint_as_float(r[8 * q4 + 2]) * inv, __uint_as_float(r[8 * q4 + 3]) * inv);
-                        v.z = pack_bf16x2(__uint_as_float(r[8 * q4 + 4]) * inv, __uint_as_float(r[8 * q4 + 5]) * inv);
-                        v.w = pack_bf16x2(__uint_as_float(r[8 * q4 + 6]) * inv, __uint_as_float(r[8 * q4 + 7]) * inv);
+                        v.x = pack_bf16x2(__uint_as_float(o[8 * q4 + 0]) * inv, __uint_as_float(o[8 * q4 + 1]) * inv);
+                        v.y = pack_bf16x2(__uint_as_float(o[8 * q4 + 2]) * inv, __uint_as_float(o[8 * q4 + 3]) * inv);
+                        v.z = pack_bf16x2(__uint_as_float(o[8 * q4 + 4]) * inv, __uint_as_float(o[8 * q4 + 5]) * inv);
+                        v.w = pack_bf16x2(__uint_as_float(o[8 * q4 + 6]) * inv, __uint_as_float(o[8 * q4 + 7]) * inv);
                         dst[q4] = v;
                     }
                 }
             }
-            if (row_valid && p.lse)
+            if (row_valid && half == 0 && p.lse)
                 p.lse[(size_t)(q0 + i0 + token) * p.num_q_heads + g * G + head] =
                     (m + __log2f(l)) * kLn2;
         }
