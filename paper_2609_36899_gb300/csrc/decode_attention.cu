@@ -78,6 +78,10 @@ __device__ __forceinline__ void append_rows(const PlanParams &p)
 
 __global__ void __launch_bounds__(1024, 1) plan_kernel(const PlanParams p)
 {
+    // Let the attention kernel launch now: it sets up its shared memory and then
+    // waits (griddepcontrol.wait) for this whole grid to finish before it reads
+    // anything the planner or the append CTAs write.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (blockIdx.x > 0) {
         append_rows(p);
         return;
@@ -279,6 +283,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             reinterpret_cast<uint4 *>(qbuf)[i] = make_uint4(0, 0, 0, 0);
     }
     __syncthreads();
+    // Everything above overlaps the planner (programmatic dependent launch);
+    // from here on the planner's and the append CTAs' writes are visible.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
 
     const long long W = p.hdr->total_work;
     const int T = p.hdr->num_slices;
@@ -723,8 +730,18 @@ cudaError_t launch_attention_d(const AttnParams &p, const CUtensorMap &kmap,
             return e;
         configured = true;
     }
-    decode_attention_kernel<D><<<grid, kAttnThreads, smem, stream>>>(p, kmap, vmap);
-    return cudaGetLastError();
+    // Programmatic dependent launch: may start while the planner still runs.
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kAttnThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, decode_attention_kernel<D>, p, kmap, vmap);
 }
 
 }  // namespace
