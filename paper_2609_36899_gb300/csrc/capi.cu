@@ -617,8 +617,10 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
     p.max_pages = max_pages;
     p.num_pages = num_pages;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
-    // upper bound on work items: sum_b ceil(C_b G / 128) <= T G / 128 + B
-    const long long grid = (long long)num_kv_heads * (batch + ((long long)total_q * group + 127) / 128);
+    // upper bound on work items: sum_b ceil(C_b G / R) <= T G / R + B, R rows per item
+    const long long rows = prefill_rows_per_item();
+    const long long grid =
+        (long long)num_kv_heads * (batch + ((long long)total_q * group + rows - 1) / rows);
     if (grid > INT32_MAX)
         return CADKV_ERR_UNSUPPORTED;
     return launch_prefill(p, qmap, kmap, vmap, (int)grid, reinterpret_cast<cudaStream_t>(stream)) ==

@@ -102,6 +102,7 @@ struct PrefillParams {
 };
 
 size_t prefill_smem_bytes();
+int prefill_rows_per_item();  // (query token, head) rows one prefill CTA handles
 cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, const CUtensorMap &kmap,
                            const CUtensorMap &vmap, int grid, cudaStream_t stream);
 

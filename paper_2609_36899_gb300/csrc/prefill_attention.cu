@@ -4,27 +4,30 @@
 // When prepared KV state cannot be used, the destination recomputes the
 // prefix (Sec. 4.4, the fallback of late-bound KV preparation): each
 // trajectory's last C_b tokens attend causally over its paged KV.  Unlike the
-// decode step this is a dense contraction (128 query rows share every key
-// tile), so it runs on tcgen05.mma:
+// decode step this is a dense contraction, so it runs on tcgen05.mma:
 //
-//  * One CTA per work item (trajectory b, KV head g, tile of 128 query rows).
-//    A row is a (query token, query head of group g) pair, token-major, so
-//    the G heads sharing a KV head share every K/V tile (GQA).
-//  * Warp 0 (TMA producer) loads the Q tile once (3-D tensor map, two 64-
-//    column panels, 128-byte swizzle) and streams K and V tiles of 128 keys
-//    (8 pages, two 2 KB boxes per page and operand, issued from 32 lanes at
-//    once) into 2-stage rings.
-//  * Warp 1 (MMA issuer, one lane) computes S_j = Q K_j^T into one of two TMEM
-//    buffers (128 lanes x 128 fp32 columns) while the softmax warps work on
-//    the other, then O += P_j V_j into a third TMEM region (V as an MN-major
-//    operand straight from the swizzled stage).
-//  * Warps 2-9 (softmax, two warpgroups; a thread owns one query row = one
-//    TMEM lane and 64 of its 128 key columns) read S_j with tcgen05.ld, apply
-//    the causal mask (only on tiles that cross the diagonal), combine the two
-//    halves' row maxima through shared memory, keep a running max (rescaling
-//    the O row in TMEM only when the max grows by more than 2^8), write P_j as
-//    bf16 into a swizzled shared-memory tile (the A operand of the PV MMA),
-//    and finally normalise O and write out and lse.
+//  * One CTA per work item (trajectory b, KV head g, 256 query rows).  A row
+//    is a (query token, query head of group g) pair, token-major, so the G
+//    heads sharing a KV head share every K/V tile (GQA).  The 256 rows form
+//    two 128-row tiles, A and B, that share each K/V tile: every K/V byte
+//    brought into shared memory feeds twice the MMA work.
+//  * Warp 0 (TMA producer) loads the two Q tiles once (3-D tensor map, two
+//    64-column panels each, 128-byte swizzle) and streams K and V tiles of 128
+//    keys (8 pages, two 2 KB boxes per page and operand, issued from 32 lanes
+//    at once) into 2-stage rings.
+//  * Warp 1 (MMA issuer, one lane) keeps S_A, S_B, O_A, O_B in TMEM (4 x 128
+//    fp32 columns).  Per key tile j it issues S_X = Q_X K_j^T and, once the
+//    softmax has turned S_X into P_X, O_X += P_X V_j with P_X read straight
+//    from TMEM (the MMA form whose A operand lives in tensor memory) and V as
+//    an MN-major operand from the swizzled stage.  Tiles A and B alternate, so
+//    the tensor cores work on one tile while the softmax works on the other.
+//  * Warps 2-5 (tile A) and 6-9 (tile B): one query row per thread = one TMEM
+//    lane.  tcgen05.ld of S (two passes over 32-column chunks), causal mask
+//    only on tiles that cross the diagonal, running max with lazy O rescaling
+//    (only when the max grows by more than 2^8; the decision is warp-uniform
+//    since tcgen05.ld/st are warp-collective), P = 2^(s - m) packed to bf16
+//    and stored with tcgen05.st over the S columns already consumed.  Finally
+//    O / l and lse.
 //  * All waits are bounded; on timeout the kernel records CADKV_ERR_TIMEOUT,
 //    waits for its own copies and MMAs, frees TMEM and returns.
 #include <cfloat>
@@ -39,24 +42,24 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr float kLn2 = 0.6931471805599453f;
-constexpr int kRows = 128;            // query rows per tile = MMA M
-constexpr int kKeys = 128;            // keys per tile = MMA N of QK^T, K of PV
-constexpr int kD = 128;               // head_dim
-constexpr int kPanel = 16384;         // 128 rows x 128 B (one 64-column panel)
-constexpr int kTileBytes = 2 * kPanel;  // 128 rows x 128 columns bf16
+constexpr int kRows = 128;               // query rows per tile = MMA M
+constexpr int kTiles = 2;                // query tiles per CTA (A and B)
+constexpr int kItemRows = kRows * kTiles;
+constexpr int kKeys = 128;               // keys per tile = MMA N of QK^T, K of PV
+constexpr int kD = 128;                  // head_dim
+constexpr int kPanel = 16384;            // 128 rows x 128 B (one 64-column panel)
+constexpr int kTileBytes = 2 * kPanel;   // 128 rows x 128 columns bf16
 constexpr int kPageBlock = kPageSize * kD * 2;  // one (page, head) block: 4 KB
-constexpr int kSoftmaxThreads = 256;  // two warpgroups, 64 key columns of every row each
+constexpr int kSoftmaxThreads = 128 * kTiles;   // one warpgroup per query tile
 constexpr int kPrefillThreads = 64 + kSoftmaxThreads;  // producer, MMA, softmax
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 struct PrefillSmem {
-    uint8_t q[kTileBytes];
-    uint8_t p[kTileBytes];
+    uint8_t q[kTiles][kTileBytes];
     uint8_t k[2][kTileBytes];
     uint8_t v[2][kTileBytes];
-    float red[2][2][kRows];  // [tile parity][half][row]: partial row maxima (sums at the end)
-    uint64_t q_full, s_full[2], p_full, o_done, k_full[2], k_empty[2], v_full[2], v_empty[2],
-        mma_done, pair;
+    uint64_t q_full, s_full[kTiles], p_full[kTiles], o_done[kTiles], k_full[2], k_empty[2],
+        v_full[2], v_empty[2], mma_done;
     uint32_t tmem_base;
     int abort;
 };
@@ -78,13 +81,25 @@ __device__ __forceinline__ uint32_t idesc_bf16(int m, int n, int a_mn, int b_mn)
            ((uint32_t)b_mn << 16) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
-__device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
-                                     uint32_t accumulate)
+// D (TMEM) = A (smem descriptor) * B (smem descriptor) [+ D]
+__device__ __forceinline__ void umma_ss(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                        uint32_t accumulate)
 {
     asm volatile(
         "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
         "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// D (TMEM) = A (TMEM: one row per lane, two bf16 per column) * B (smem) [+ D]
+__device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b,
+                                        uint32_t idesc, uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(idesc), "r"(accumulate)
         : "memory");
 }
 
@@ -121,6 +136,14 @@ __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::
                  "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])             \
                  : "memory")
 
+#define CADKV_TMEM_ST16(taddr, r)                                                                   \
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,"    \
+                 "%11,%12,%13,%14,%15,%16};" ::"r"(taddr),                                        \
+                 "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]),       \
+                 "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]),   \
+                 "r"(r[14]), "r"(r[15])                                                           \
+                 : "memory")
+
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
@@ -132,7 +155,6 @@ __global__ void __launch_bounds__(1024, 1) prefill_plan_kernel(const PrefillPara
     __shared__ long long warp_sums[32];
     __shared__ long long carry_s;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int rows_per_token = p.group;
     if (tid == 0) {
         p.hdr->status = 0;
         carry_s = 0;
@@ -149,7 +171,7 @@ __global__ void __launch_bounds__(1024, 1) prefill_plan_kernel(const PrefillPara
                 n > p.max_pages * kPageSize) {
                 record_status(&p.hdr->status, CADKV_ERR_SHAPE);
             } else {
-                items = (long long)p.num_kv_heads * ((c * rows_per_token + kRows - 1) / kRows);
+                items = (long long)p.num_kv_heads * ((c * p.group + kItemRows - 1) / kItemRows);
             }
         }
         long long v = items;
@@ -203,7 +225,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
     if (item >= total)
         return;  // uniform across the CTA, before any barrier or TMEM use
 
-    // ---- decode the work item: (trajectory b, KV head g, query tile qt)
+    // ---- decode the work item: (trajectory b, KV head g, 256-row query block qt)
     int lo = 0, hi = p.batch - 1;
     while (lo < hi) {  // largest b with item_prefix[b] <= item
         const int mid = (lo + hi + 1) >> 1;
@@ -218,12 +240,12 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
     const long long q0 = p.q_offsets[b];
     const int chunk = (int)(p.q_offsets[b + 1] - q0);
     const int n = p.context_lens[b];
-    const int qtiles = (chunk * G + kRows - 1) / kRows;
+    const int qblocks = (chunk * G + kItemRows - 1) / kItemRows;
     const int local = (int)(item - p.item_prefix[b]);
-    const int g = local / qtiles;
-    const int qt = qtiles - 1 - local % qtiles;  // heaviest tiles first
-    const int i0 = qt * tokens_per_tile;
-    const int valid_tokens = min(tokens_per_tile, chunk - i0);
+    const int g = local / qblocks;
+    const int qt = qblocks - 1 - local % qblocks;  // heaviest blocks first
+    const int i0 = qt * kTiles * tokens_per_tile;  // first token of tile A
+    const int valid_tokens = min(kTiles * tokens_per_tile, chunk - i0);
     const int chunk_start = n - chunk;
     const int pos_max = chunk_start + i0 + valid_tokens - 1;
     const int num_kt = (pos_max + 1 + kKeys - 1) / kKeys;
@@ -231,11 +253,11 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
 
     if (tid == 0) {
         mbar_init(&sm.q_full, 1);
-        mbar_init(&sm.s_full[0], 1);
-        mbar_init(&sm.s_full[1], 1);
-        mbar_init(&sm.p_full, kSoftmaxThreads);
-        mbar_init(&sm.pair, kSoftmaxThreads);
-        mbar_init(&sm.o_done, 1);
+        for (int t = 0; t < kTiles; ++t) {
+            mbar_init(&sm.s_full[t], 1);
+            mbar_init(&sm.p_full[t], 128);
+            mbar_init(&sm.o_done[t], 1);
+        }
         for (int s = 0; s < 2; ++s) {
             mbar_init(&sm.k_full[s], 1);
             mbar_init(&sm.k_empty[s], 1);
@@ -256,30 +278,28 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = sm.tmem_base;
-    const uint32_t tmem_s[2] = {tmem, tmem + 128};
-    const uint32_t tmem_o = tmem + 256;
+    // columns: S_A [0,128), S_B [128,256), O_A [256,384), O_B [384,512); P_X is
+    // written over the first 64 columns of S_X (two bf16 per column).
     volatile int *abort_flag = &sm.abort;
 
     if (warp == 0) {
         // ============================ TMA producer ============================
-        // Q: one 3-D tensor-map load (two 64-column panels).  K, V: a tile's 8
-        // pages as 2 KB boxes (16 tokens x one 64-column panel) landing in the
-        // panel layout the MMAs read (row = key).  Lane 0 waits for free stages
-        // and arms the barriers; then all 32 lanes issue one box each (lanes
-        // 0-15: K, 16-31: V; page = (lane/2)%8, panel = lane%2) so a tile's 32
-        // copies start together.
         bool ok = true;
         int issued = 0;
-        const uint64_t policy = l2_evict_first_policy();
+        // every (trajectory, KV head)'s K/V is re-read by all its query-block CTAs
+        const uint64_t policy = l2_evict_last_policy();
         if (lane == 0) {
             prefetch_tensor_map(&qmap);
             prefetch_tensor_map(&kmap);
             prefetch_tensor_map(&vmap);
-            mbar_arrive_expect_tx(&sm.q_full, kTileBytes);
-            const int qy = (int)(q0 + i0);
-            for (int h = 0; h < 2; ++h)
-                tma_load_3d(sm.q + h * kPanel, &qmap, h * 64, g * G, qy, &sm.q_full);
+            mbar_arrive_expect_tx(&sm.q_full, kTiles * kTileBytes);
+            for (int t = 0; t < kTiles; ++t) {
+                const int qy = (int)(q0 + i0 + t * tokens_per_tile);
+                for (int h = 0; h < 2; ++h)
+                    tma_load_3d(sm.q[t] + h * kPanel, &qmap, h * 64, g * G, qy, &sm.q_full);
+            }
         }
+        // lanes 0-15: K, 16-31: V; page = (lane / 2) % 8, 64-column panel = lane % 2
         const int op = lane >> 4, pg = (lane >> 1) & 7, hh = lane & 1;
         for (int j = 0; j < num_kt; ++j) {
             const int s = j & 1;
@@ -329,46 +349,58 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
         if (lane == 0) {
             const uint32_t id_qk = idesc_bf16(kRows, kKeys, 0, 0);
             const uint32_t id_pv = idesc_bf16(kRows, kD, 0, 1);
-            bool ok = mbar_wait(&sm.q_full, 0, abort_flag) && mbar_wait(&sm.k_full[0], 0, abort_flag);
-            auto issue_qk = [&](int j) {
+            auto issue_s = [&](int t, int j) {  // S_t = Q_t K_j^T
                 const int s = j & 1;
-                tc_fence_after();
 #pragma unroll
                 for (int k = 0; k < kD / 16; ++k) {
                     const int atom = k >> 2, kin = k & 3;
-                    const uint64_t a = desc_sw128(smem_addr(sm.q + atom * kPanel) + kin * 32, 16, 1024);
+                    const uint64_t a = desc_sw128(smem_addr(sm.q[t] + atom * kPanel) + kin * 32, 16, 1024);
                     const uint64_t bd = desc_sw128(smem_addr(sm.k[s] + atom * kPanel) + kin * 32, 16, 1024);
-                    umma(tmem_s[s], a, bd, id_qk, k > 0);
+                    umma_ss(tmem + t * kRows, a, bd, id_qk, k > 0);
                 }
-                umma_commit(&sm.s_full[s]);
-                umma_commit(&sm.k_empty[s]);  // K_j is read only by S_j: free it early
+                umma_commit(&sm.s_full[t]);
             };
-            if (ok)
-                issue_qk(0);
+            auto issue_pv = [&](int t, int j) {  // O_t += P_t V_j, P_t from TMEM
+                const int s = j & 1;
+#pragma unroll
+                for (int k = 0; k < kKeys / 16; ++k) {  // keys 16k .. 16k+15 = P columns 8k ..
+                    const uint64_t bd = desc_sw128(smem_addr(sm.v[s]) + k * 2048, kPanel, 1024);
+                    umma_ts(tmem + 256 + t * kRows, tmem + t * kRows + 8 * k, bd, id_pv,
+                            (j > 0 || k > 0) ? 1u : 0u);
+                }
+                umma_commit(&sm.o_done[t]);
+            };
+            bool ok = mbar_wait(&sm.q_full, 0, abort_flag) && mbar_wait(&sm.k_full[0], 0, abort_flag);
+            if (ok) {
+                tc_fence_after();
+                issue_s(0, 0);
+                issue_s(1, 0);
+                umma_commit(&sm.k_empty[0]);
+            }
             for (int j = 0; j < num_kt && ok; ++j) {
                 const int s = j & 1;
-                if (j + 1 < num_kt) {
-                    ok = mbar_wait(&sm.k_full[(j + 1) & 1], ((j + 1) >> 1) & 1, abort_flag);
-                    if (!ok)
-                        break;
-                    issue_qk(j + 1);  // S buffer (j+1)&1 was released with P_{j-1}
-                }
-                ok = mbar_wait(&sm.p_full, j & 1, abort_flag) &&
-                     mbar_wait(&sm.v_full[s], (j >> 1) & 1, abort_flag);
+                const bool more = j + 1 < num_kt;
+                // tile A: PV_A(j) once P_A(j) is in TMEM, then S_A(j+1) over it
+                ok = mbar_wait(&sm.p_full[0], j & 1, abort_flag) &&
+                     mbar_wait(&sm.v_full[s], (j >> 1) & 1, abort_flag) &&
+                     (!more || mbar_wait(&sm.k_full[(j + 1) & 1], ((j + 1) >> 1) & 1, abort_flag));
                 if (!ok)
                     break;
                 tc_fence_after();
-                // O += P V: V as an MN-major operand (64-column panels 16 KB apart,
-                // 8-key groups 1 KB apart); K step k = keys 16k .. 16k+15.
-#pragma unroll
-                for (int k = 0; k < kKeys / 16; ++k) {
-                    const int atom = k >> 2, kin = k & 3;
-                    const uint64_t a = desc_sw128(smem_addr(sm.p + atom * kPanel) + kin * 32, 16, 1024);
-                    const uint64_t bd = desc_sw128(smem_addr(sm.v[s]) + k * 2048, kPanel, 1024);
-                    umma(tmem_o, a, bd, id_pv, (j > 0 || k > 0) ? 1u : 0u);
-                }
-                umma_commit(&sm.o_done);
+                issue_pv(0, j);
+                if (more)
+                    issue_s(0, j + 1);
+                // tile B likewise; then V_j and K_{j+1} are no longer needed
+                ok = mbar_wait(&sm.p_full[1], j & 1, abort_flag);
+                if (!ok)
+                    break;
+                tc_fence_after();
+                issue_pv(1, j);
                 umma_commit(&sm.v_empty[s]);
+                if (more) {
+                    issue_s(1, j + 1);
+                    umma_commit(&sm.k_empty[(j + 1) & 1]);
+                }
             }
             if (!ok) {
                 *abort_flag = 1;
@@ -382,142 +414,113 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
         __syncwarp();
     } else {
         // ============================ softmax warps ============================
-        // Warp w (2..9) owns TMEM lane quarter w % 4 (rows 32*(w%4) ..) and key
-        // columns 64*half .. 64*half+63 of every tile, half = (w - 2) / 4.  The two
-        // halves of a row combine their maxima through shared memory.
-        const int half = (warp - 2) >> 2;
-        const int row = 32 * (warp & 3) + lane;  // TMEM lane = query row
+        const int t = (warp - 2) >> 2;            // query tile: 0 (A) or 1 (B)
+        const int row = 32 * (warp & 3) + lane;   // TMEM lane = row of the tile
         const uint32_t lane_base = (uint32_t)(32 * (warp & 3)) << 16;
-        const uint32_t col0 = 64u * half;
-        const int token = row / G, head = row % G;
+        const uint32_t s_col = tmem + lane_base + t * kRows;
+        const uint32_t o_col = tmem + lane_base + 256 + t * kRows;
+        const int token = t * tokens_per_tile + row / G, head = row % G;
         const bool row_valid = token < valid_tokens;
         const int pos_row = row_valid ? chunk_start + i0 + token : pos_max;
-        const int pos_min = chunk_start + i0;  // smallest position of any row in the tile
+        const int pos_min = chunk_start + i0 + t * tokens_per_tile;  // first row of the tile
         const float scale = p.scale_log2;
         float m = -INFINITY, l = 0.f;
-        uint32_t pair_phase = 0;
         bool ok = true;
-        uint8_t *prow = sm.p + half * kPanel + row * 128;
-        auto pair_sync = [&]() {
-            mbar_arrive(&sm.pair);
-            const bool done = mbar_wait(&sm.pair, pair_phase, abort_flag);
-            pair_phase ^= 1u;
-            return __all_sync(kFull, done);
-        };
         for (int j = 0; j < num_kt && ok; ++j) {
-            const int s = j & 1;
-            ok = __all_sync(kFull, mbar_wait(&sm.s_full[s], (j >> 1) & 1, abort_flag));
+            ok = __all_sync(kFull, mbar_wait(&sm.s_full[t], j & 1, abort_flag));
             if (!ok)
                 break;
             tc_fence_after();
-            const int key0 = j * kKeys + (int)col0;
-            // keys key0 .. key0+63 are all visible to every row of the tile?
-            const bool full_tile = key0 + 63 <= pos_min;
-            uint32_t r[64];
-            CADKV_TMEM_LD32(tmem_s[s] + lane_base + col0, r);
-            CADKV_TMEM_LD32(tmem_s[s] + lane_base + col0 + 32, (r + 32));
-            tmem_wait_ld();
-            float x[64];
+            const int key0 = j * kKeys;
+            const bool full_tile = key0 + kKeys - 1 <= pos_min;  // no key masked for any row
+            // pass 1: masked row max
             float mx = -INFINITY;
-            if (full_tile) {
+            for (int c = 0; c < 4; ++c) {
+                uint32_t r[32];
+                CADKV_TMEM_LD32(s_col + c * 32, r);
+                tmem_wait_ld();
+                if (full_tile) {
 #pragma unroll
-                for (int e = 0; e < 64; ++e) {
-                    x[e] = __uint_as_float(r[e]) * scale;
-                    mx = fmaxf(mx, x[e]);
-                }
-            } else {
+                    for (int e = 0; e < 32; ++e)
+                        mx = fmaxf(mx, __uint_as_float(r[e]));
+                } else {
 #pragma unroll
-                for (int e = 0; e < 64; ++e) {
-                    x[e] = key0 + e <= pos_row ? __uint_as_float(r[e]) * scale : -INFINITY;
-                    mx = fmaxf(mx, x[e]);
+                    for (int e = 0; e < 32; ++e)
+                        if (key0 + c * 32 + e <= pos_row)
+                            mx = fmaxf(mx, __uint_as_float(r[e]));
                 }
             }
-            sm.red[s][half][row] = mx;
-            ok = pair_sync();
-            if (!ok)
-                break;
-            mx = fmaxf(mx, sm.red[s][half ^ 1][row]);
-            const float m_new = fmaxf(m, mx);
-            // P smem and O are free once the previous PV has completed
-            if (j > 0) {
-                ok = __all_sync(kFull, mbar_wait(&sm.o_done, (j - 1) & 1, abort_flag));
-                if (!ok)
-                    break;
-                tc_fence_after();
-            }
-            // tcgen05.ld/st are warp-collective: the whole warp rescales when any
-            // lane's max grew past the threshold (rescaling to the true max is
-            // always correct, only skipping it needs the bound).  Both halves of a
-            // row see the same maxima, so they take the same decision.
+            const float m_new = fmaxf(m, mx * scale);
+            // S_t(j) was issued after PV_t(j-1), so O_t is stable here.
             if (__any_sync(kFull, m_new > m + kRescaleThreshold)) {
                 const float alpha = exp2_approx(m - m_new);  // 0 on the first tile
                 if (j > 0) {
-                    for (int c = 0; c < 2; ++c) {
+                    for (int c = 0; c < 4; ++c) {
                         uint32_t o[32];
-                        CADKV_TMEM_LD32(tmem_o + lane_base + col0 + c * 32, o);
+                        CADKV_TMEM_LD32(o_col + c * 32, o);
                         tmem_wait_ld();
 #pragma unroll
                         for (int e = 0; e < 32; ++e)
                             o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-                        CADKV_TMEM_ST32(tmem_o + lane_base + col0 + c * 32, o);
+                        CADKV_TMEM_ST32(o_col + c * 32, o);
                     }
-                    tmem_wait_st();
                 }
                 l *= alpha;
                 m = m_new;
             }
-            // P = 2^(x - m) as bf16: keys col0 .. col0+63 are panel `half` of the row
+            // pass 2: P = 2^(s*scale - m) as bf16 pairs over S columns already read
+            for (int c = 0; c < 4; ++c) {
+                uint32_t r[32];
+                CADKV_TMEM_LD32(s_col + c * 32, r);
+                tmem_wait_ld();
+                uint32_t packed[16];
 #pragma unroll
-            for (int cin = 0; cin < 8; ++cin) {
-                uint32_t packed[4];
-#pragma unroll
-                for (int e2 = 0; e2 < 4; ++e2) {
-                    const float p0 = exp2_approx(x[8 * cin + 2 * e2] - m);
-                    const float p1 = exp2_approx(x[8 * cin + 2 * e2 + 1] - m);
+                for (int e = 0; e < 32; e += 2) {
+                    float p0, p1;
+                    if (full_tile) {
+                        p0 = exp2_approx(__uint_as_float(r[e]) * scale - m);
+                        p1 = exp2_approx(__uint_as_float(r[e + 1]) * scale - m);
+                    } else {
+                        const int key = key0 + c * 32 + e;
+                        p0 = key <= pos_row ? exp2_approx(__uint_as_float(r[e]) * scale - m) : 0.f;
+                        p1 = key + 1 <= pos_row ? exp2_approx(__uint_as_float(r[e + 1]) * scale - m) : 0.f;
+                    }
                     l += p0 + p1;
-                    packed[e2] = pack_bf16x2(p0, p1);
+                    packed[e >> 1] = pack_bf16x2(p0, p1);
                 }
-                *reinterpret_cast<uint4 *>(prow + ((cin ^ (row & 7)) << 4)) =
-                    make_uint4(packed[0], packed[1], packed[2], packed[3]);
+                CADKV_TMEM_ST16(s_col + c * 16, packed);
             }
-            if (j == num_kt - 1) {
+            tmem_wait_st();
+            if (j == num_kt - 1 && t == 0) {
                 // Zero V rows past pos_max: those keys may hold NaN (slots past n_b,
-                // or pages never loaded) and 0 * NaN would poison the PV sum.
-                ok = __all_sync(kFull, mbar_wait(&sm.v_full[s], (j >> 1) & 1, abort_flag));
+                // or pages never loaded) and 0 * NaN would poison the PV sums.
+                ok = __all_sync(kFull, mbar_wait(&sm.v_full[j & 1], (j >> 1) & 1, abort_flag));
                 if (!ok)
                     break;
-                const int t = tid - 64;                    // 0..255
-                const int key_row = t & 127, hv = t >> 7;
-                if (j * kKeys + key_row > pos_max) {
-                    uint4 *rz = reinterpret_cast<uint4 *>(sm.v[s] + hv * kPanel + key_row * 128);
+                if (key0 + row > pos_max) {
+                    for (int h = 0; h < 2; ++h) {
+                        uint4 *rz = reinterpret_cast<uint4 *>(sm.v[j & 1] + h * kPanel + row * 128);
 #pragma unroll
-                    for (int c16 = 0; c16 < 8; ++c16)
-                        rz[c16] = make_uint4(0, 0, 0, 0);
+                        for (int c16 = 0; c16 < 8; ++c16)
+                            rz[c16] = make_uint4(0, 0, 0, 0);
+                    }
                 }
+                fence_proxy_async_smem();
             }
-            fence_proxy_async_smem();
             tc_fence_before();
-            mbar_arrive(&sm.p_full);
+            mbar_arrive(&sm.p_full[t]);
         }
-        // ---- epilogue: combine the two halves' sums, O / l -> out, lse
+        // ---- epilogue: O / l -> out, lse
         if (ok) {
-            // the last tile's maxima have been read by both halves (both passed the
-            // pair barrier of that tile), so parity slot 0/1 of the last tile is free
-            sm.red[num_kt & 1][half][row] = l;
-            ok = pair_sync();
-        }
-        if (ok) {
-            l += sm.red[num_kt & 1][half ^ 1][row];
-            ok = __all_sync(kFull, mbar_wait(&sm.o_done, (num_kt - 1) & 1, abort_flag));
+            ok = __all_sync(kFull, mbar_wait(&sm.o_done[t], (num_kt - 1) & 1, abort_flag));
             tc_fence_after();
         }
         if (ok) {
             const float inv = 1.f / l;
-            __nv_bfloat16 *orow =
-                p.out + ((size_t)(q0 + i0 + token) * p.num_q_heads + g * G + head) * kD + col0;
-            for (int c = 0; c < 2; ++c) {
+            __nv_bfloat16 *orow = p.out + ((size_t)(q0 + i0 + token) * p.num_q_heads + g * G + head) * kD;
+            for (int c = 0; c < 4; ++c) {
                 uint32_t o[32];
-                CADKV_TMEM_LD32(tmem_o + lane_base + col0 + c * 32, o);
+                CADKV_TMEM_LD32(o_col + c * 32, o);
                 tmem_wait_ld();
                 if (row_valid) {
                     uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
@@ -532,7 +535,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                     }
                 }
             }
-            if (row_valid && half == 0 && p.lse)
+            if (row_valid && p.lse)
                 p.lse[(size_t)(q0 + i0 + token) * p.num_q_heads + g * G + head] =
                     (m + __log2f(l)) * kLn2;
         }
@@ -553,6 +556,8 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
 }  // namespace
 
 size_t prefill_smem_bytes() { return sizeof(PrefillSmem) + 1024; }
+
+int prefill_rows_per_item() { return kItemRows; }
 
 cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, const CUtensorMap &kmap,
                            const CUtensorMap &vmap, int grid, cudaStream_t stream)

@@ -108,6 +108,14 @@ __device__ __forceinline__ uint64_t l2_evict_first_policy()
     return policy;
 }
 
+// L2 policy that keeps lines resident preferentially (data other CTAs re-read).
+__device__ __forceinline__ uint64_t l2_evict_last_policy()
+{
+    uint64_t policy;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(policy));
+    return policy;
+}
+
 // 2-D tiled tensor copy global -> shared through tensor map `map` at
 // coordinates (x inner, y outer), with an L2 cache-eviction hint.
 __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int x, int y,
