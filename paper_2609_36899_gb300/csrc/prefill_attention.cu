@@ -22,7 +22,7 @@
 //    an MN-major operand from the swizzled stage.  Tiles A and B alternate, so
 //    the tensor cores work on one tile while the softmax works on the other.
 //  * Warps 2-5 (tile A) and 6-9 (tile B): one query row per thread = one TMEM
-//    lane.  tcgen05.ld of S (two passes over 32-column chunks), causal mask
+//    lane.  The row's 128 scores come in one burst of tcgen05.ld, causal mask
 //    only on tiles that cross the diagonal, running max with lazy O rescaling
 //    (only when the max grows by more than 2^8; the decision is warp-uniform
 //    since tcgen05.ld/st are warp-collective), P = 2^(s - m) packed to bf16
@@ -433,23 +433,23 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             tc_fence_after();
             const int key0 = j * kKeys;
             const bool full_tile = key0 + kKeys - 1 <= pos_min;  // no key masked for any row
-            // pass 1: masked row max
-            float mx = -INFINITY;
-            for (int c = 0; c < 4; ++c) {
-                uint32_t r[32];
-                CADKV_TMEM_LD32(s_col + c * 32, r);
-                tmem_wait_ld();
-                if (full_tile) {
+            // the row's 128 scores in one burst of loads, one wait
+            uint32_t r[kKeys];
+            CADKV_TMEM_LD32(s_col + 0, r);
+            CADKV_TMEM_LD32(s_col + 32, (r + 32));
+            CADKV_TMEM_LD32(s_col + 64, (r + 64));
+            CADKV_TMEM_LD32(s_col + 96, (r + 96));
+            tmem_wait_ld();
+            if (!full_tile) {  // causal mask on tiles that cross the diagonal
 #pragma unroll
-                    for (int e = 0; e < 32; ++e)
-                        mx = fmaxf(mx, __uint_as_float(r[e]));
-                } else {
-#pragma unroll
-                    for (int e = 0; e < 32; ++e)
-                        if (key0 + c * 32 + e <= pos_row)
-                            mx = fmaxf(mx, __uint_as_float(r[e]));
-                }
+                for (int e = 0; e < kKeys; ++e)
+                    if (key0 + e > pos_row)
+                        r[e] = __float_as_uint(-INFINITY);
             }
+            float mx = -INFINITY;
+#pragma unroll
+            for (int e = 0; e < kKeys; ++e)
+                mx = fmaxf(mx, __uint_as_float(r[e]));
             const float m_new = fmaxf(m, mx * scale);
             // S_t(j) was issued after PV_t(j-1), so O_t is stable here.
             if (__any_sync(kFull, m_new > m + kRescaleThreshold)) {
@@ -468,23 +468,15 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                 l *= alpha;
                 m = m_new;
             }
-            // pass 2: P = 2^(s*scale - m) as bf16 pairs over S columns already read
+            // P = 2^(s*scale - m) as bf16 pairs, over S columns already read
+            // (masked scores are -inf, so their P is exactly 0)
+#pragma unroll
             for (int c = 0; c < 4; ++c) {
-                uint32_t r[32];
-                CADKV_TMEM_LD32(s_col + c * 32, r);
-                tmem_wait_ld();
                 uint32_t packed[16];
 #pragma unroll
                 for (int e = 0; e < 32; e += 2) {
-                    float p0, p1;
-                    if (full_tile) {
-                        p0 = exp2_approx(__uint_as_float(r[e]) * scale - m);
-                        p1 = exp2_approx(__uint_as_float(r[e + 1]) * scale - m);
-                    } else {
-                        const int key = key0 + c * 32 + e;
-                        p0 = key <= pos_row ? exp2_approx(__uint_as_float(r[e]) * scale - m) : 0.f;
-                        p1 = key + 1 <= pos_row ? exp2_approx(__uint_as_float(r[e + 1]) * scale - m) : 0.f;
-                    }
+                    const float p0 = exp2_approx(__uint_as_float(r[32 * c + e]) * scale - m);
+                    const float p1 = exp2_approx(__uint_as_float(r[32 * c + e + 1]) * scale - m);
                     l += p0 + p1;
                     packed[e >> 1] = pack_bf16x2(p0, p1);
                 }
