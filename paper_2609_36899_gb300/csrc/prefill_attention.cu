@@ -451,20 +451,11 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             for (int e = 0; e < kKeys; ++e)
                 mx = fmaxf(mx, __uint_as_float(r[e]));
             const float m_new = fmaxf(m, mx * scale);
-            // S_t(j) was issued after PV_t(j-1), so O_t is stable here.
-            if (__any_sync(kFull, m_new > m + kRescaleThreshold)) {
-                const float alpha = exp2_approx(m - m_new);  // 0 on the first tile
-                if (j > 0) {
-                    for (int c = 0; c < 4; ++c) {
-                        uint32_t o[32];
-                        CADKV_TMEM_LD32(o_col + c * 32, o);
-                        tmem_wait_ld();
-#pragma unroll
-                        for (int e = 0; e < 32; ++e)
-                            o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-                        CADKV_TMEM_ST32(o_col + c * 32, o);
-                    }
-                }
+            // Lazy rescaling: keep the stale max unless some lane's grew past the
+            // threshold; the decision is warp-uniform (tcgen05.ld/st are collective).
+            const bool rescale = __any_sync(kFull, m_new > m + kRescaleThreshold);
+            const float alpha = rescale ? exp2_approx(m - m_new) : 1.f;  // 0 on the first tile
+            if (rescale) {
                 l *= alpha;
                 m = m_new;
             }
@@ -481,6 +472,19 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                     packed[e >> 1] = pack_bf16x2(p0, p1);
                 }
                 CADKV_TMEM_ST16(s_col + c * 16, packed);
+            }
+            // O_t is stable here (S_t(j) was issued after PV_t(j-1)) and is not read
+            // again before PV_t(j), which waits for this tile's p_full.
+            if (rescale && j > 0) {
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t o[32];
+                    CADKV_TMEM_LD32(o_col + c * 32, o);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int e = 0; e < 32; ++e)
+                        o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+                    CADKV_TMEM_ST32(o_col + c * 32, o);
+                }
             }
             tmem_wait_st();
             if (j == num_kt - 1 && t == 0) {
