@@ -14,7 +14,8 @@
 //  * Warp 0 (TMA producer) loads the two Q tiles once (3-D tensor map, two
 //    64-column panels each, 128-byte swizzle) and streams K and V tiles of 128
 //    keys (8 pages, two 2 KB boxes per page and operand, issued from 32 lanes
-//    at once) into 2-stage rings.
+//    at once) into a 3-stage K ring and a 2-stage V ring; K is released as
+//    soon as both S MMAs have read it, so it is loaded a tile ahead of V.
 //  * Warp 1 (MMA issuer, one lane) keeps S_A, S_B, O_A, O_B in TMEM (4 x 128
 //    fp32 columns).  Per key tile j it issues S_X = Q_X K_j^T and, once the
 //    softmax has turned S_X into P_X, O_X += P_X V_j with P_X read straight
@@ -53,13 +54,15 @@ constexpr int kPageBlock = kPageSize * kD * 2;  // one (page, head) block: 4 KB
 constexpr int kSoftmaxThreads = 128 * kTiles;   // one warpgroup per query tile
 constexpr int kPrefillThreads = 64 + kSoftmaxThreads;  // producer, MMA, softmax
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
+constexpr int kKStages = 3;              // K is freed early (after S), so it runs further ahead
+constexpr int kVStages = 2;
 
 struct PrefillSmem {
     uint8_t q[kTiles][kTileBytes];
-    uint8_t k[2][kTileBytes];
-    uint8_t v[2][kTileBytes];
-    uint64_t q_full, s_full[kTiles], p_full[kTiles], o_done[kTiles], k_full[2], k_empty[2],
-        v_full[2], v_empty[2], mma_done;
+    uint8_t k[kKStages][kTileBytes];
+    uint8_t v[kVStages][kTileBytes];
+    uint64_t q_full, s_full[kTiles], p_full[kTiles], o_done[kTiles], k_full[kKStages],
+        k_empty[kKStages], v_full[kVStages], v_empty[kVStages], mma_done;
     uint32_t tmem_base;
     int abort;
 };
@@ -258,9 +261,11 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             mbar_init(&sm.p_full[t], 128);
             mbar_init(&sm.o_done[t], 1);
         }
-        for (int s = 0; s < 2; ++s) {
+        for (int s = 0; s < kKStages; ++s) {
             mbar_init(&sm.k_full[s], 1);
             mbar_init(&sm.k_empty[s], 1);
+        }
+        for (int s = 0; s < kVStages; ++s) {
             mbar_init(&sm.v_full[s], 1);
             mbar_init(&sm.v_empty[s], 1);
         }
@@ -285,7 +290,6 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
     if (warp == 0) {
         // ============================ TMA producer ============================
         bool ok = true;
-        int issued = 0;
         // every (trajectory, KV head)'s K/V is re-read by all its query-block CTAs
         const uint64_t policy = l2_evict_last_policy();
         if (lane == 0) {
@@ -299,36 +303,51 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                     tma_load_3d(sm.q[t] + h * kPanel, &qmap, h * 64, g * G, qy, &sm.q_full);
             }
         }
-        // lanes 0-15: K, 16-31: V; page = (lane / 2) % 8, 64-column panel = lane % 2
+        // Step J issues K_J (lanes 0-15) and V_{J-1} (lanes 16-31): K is freed
+        // right after the S MMAs while V waits for PV, so each stream is gated
+        // only by its own ring and K runs a tile ahead.  Box = one 64-column
+        // panel of one page: page = (lane / 2) % 8, panel = lane % 2.
         const int op = lane >> 4, pg = (lane >> 1) & 7, hh = lane & 1;
-        for (int j = 0; j < num_kt; ++j) {
-            const int s = j & 1;
-            const int first_page = j * (kKeys / kPageSize);
-            const int pages = min(kKeys / kPageSize, last_page + 1 - first_page);
+        int issued_k = 0, issued_v = 0;
+        for (int J = 0; J <= num_kt && ok; ++J) {
+            const int jk = J, jv = J - 1;
+            const bool do_k = jk < num_kt, do_v = jv >= 0;
+            const int pages_k = do_k ? min(kKeys / kPageSize, last_page + 1 - jk * (kKeys / kPageSize)) : 0;
+            const int pages_v = do_v ? min(kKeys / kPageSize, last_page + 1 - jv * (kKeys / kPageSize)) : 0;
             if (lane == 0) {
-                if (j >= 2)
-                    ok = mbar_wait(&sm.k_empty[s], ((j >> 1) + 1) & 1, abort_flag) &&
-                         mbar_wait(&sm.v_empty[s], ((j >> 1) + 1) & 1, abort_flag);
-                if (ok) {
-                    mbar_arrive_expect_tx(&sm.k_full[s], (uint32_t)pages * kPageBlock);
-                    mbar_arrive_expect_tx(&sm.v_full[s], (uint32_t)pages * kPageBlock);
+                if (do_k) {
+                    const int sk = jk % kKStages;
+                    if (jk >= kKStages)
+                        ok = mbar_wait(&sm.k_empty[sk], ((jk / kKStages) + 1) & 1, abort_flag);
+                    if (ok)
+                        mbar_arrive_expect_tx(&sm.k_full[sk], (uint32_t)pages_k * kPageBlock);
+                }
+                if (do_v && ok) {
+                    const int sv = jv % kVStages;
+                    if (jv >= kVStages)
+                        ok = mbar_wait(&sm.v_empty[sv], ((jv / kVStages) + 1) & 1, abort_flag);
+                    if (ok)
+                        mbar_arrive_expect_tx(&sm.v_full[sv], (uint32_t)pages_v * kPageBlock);
                 }
             }
             ok = __shfl_sync(kFull, ok ? 1 : 0, 0) != 0;
             if (!ok)
                 break;
-            if (pg < pages) {
-                int phys = p.block_table[(size_t)b * p.max_pages + first_page + pg];
+            const int jt = op == 0 ? jk : jv;
+            const int pages = op == 0 ? pages_k : pages_v;
+            if ((op == 0 ? do_k : do_v) && pg < pages) {
+                int phys = p.block_table[(size_t)b * p.max_pages + jt * (kKeys / kPageSize) + pg];
                 if (phys < 0 || phys >= p.num_pages) {
                     record_status(&p.hdr->status, CADKV_ERR_OOB);
                     phys = 0;
                 }
                 const int y = (phys * p.num_kv_heads + g) * kPageSize;
-                uint8_t *dst = (op == 0 ? sm.k[s] : sm.v[s]) + hh * kPanel + pg * 2048;
+                uint8_t *dst = (op == 0 ? sm.k[jt % kKStages] : sm.v[jt % kVStages]) + hh * kPanel + pg * 2048;
                 tma_load_2d(dst, op == 0 ? &kmap : &vmap, hh * 64, y,
-                            op == 0 ? &sm.k_full[s] : &sm.v_full[s], policy);
+                            op == 0 ? &sm.k_full[jt % kKStages] : &sm.v_full[jt % kVStages], policy);
             }
-            ++issued;
+            issued_k += do_k;
+            issued_v += do_v;
         }
         if (lane == 0) {
             if (!ok) {
@@ -338,10 +357,10 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             // every copy this warp started must land before the CTA exits
             volatile int never = 0;
             mbar_wait(&sm.q_full, 0, &never);
-            for (int j = max(0, issued - 2); j < issued; ++j) {
-                mbar_wait(&sm.k_full[j & 1], (j >> 1) & 1, &never);
-                mbar_wait(&sm.v_full[j & 1], (j >> 1) & 1, &never);
-            }
+            for (int j = max(0, issued_k - kKStages); j < issued_k; ++j)
+                mbar_wait(&sm.k_full[j % kKStages], (j / kKStages) & 1, &never);
+            for (int j = max(0, issued_v - kVStages); j < issued_v; ++j)
+                mbar_wait(&sm.v_full[j % kVStages], (j / kVStages) & 1, &never);
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -350,7 +369,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             const uint32_t id_qk = idesc_bf16(kRows, kKeys, 0, 0);
             const uint32_t id_pv = idesc_bf16(kRows, kD, 0, 1);
             auto issue_s = [&](int t, int j) {  // S_t = Q_t K_j^T
-                const int s = j & 1;
+                const int s = j % kKStages;
 #pragma unroll
                 for (int k = 0; k < kD / 16; ++k) {
                     const int atom = k >> 2, kin = k & 3;
@@ -361,7 +380,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                 umma_commit(&sm.s_full[t]);
             };
             auto issue_pv = [&](int t, int j) {  // O_t += P_t V_j, P_t from TMEM
-                const int s = j & 1;
+                const int s = j % kVStages;
 #pragma unroll
                 for (int k = 0; k < kKeys / 16; ++k) {  // keys 16k .. 16k+15 = P columns 8k ..
                     const uint64_t bd = desc_sw128(smem_addr(sm.v[s]) + k * 2048, kPanel, 1024);
@@ -378,12 +397,13 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                 umma_commit(&sm.k_empty[0]);
             }
             for (int j = 0; j < num_kt && ok; ++j) {
-                const int s = j & 1;
+                const int sv = j % kVStages;
+                const int sk1 = (j + 1) % kKStages;
                 const bool more = j + 1 < num_kt;
                 // tile A: PV_A(j) once P_A(j) is in TMEM, then S_A(j+1) over it
                 ok = mbar_wait(&sm.p_full[0], j & 1, abort_flag) &&
-                     mbar_wait(&sm.v_full[s], (j >> 1) & 1, abort_flag) &&
-                     (!more || mbar_wait(&sm.k_full[(j + 1) & 1], ((j + 1) >> 1) & 1, abort_flag));
+                     mbar_wait(&sm.v_full[sv], (j / kVStages) & 1, abort_flag) &&
+                     (!more || mbar_wait(&sm.k_full[sk1], ((j + 1) / kKStages) & 1, abort_flag));
                 if (!ok)
                     break;
                 tc_fence_after();
@@ -396,10 +416,10 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                     break;
                 tc_fence_after();
                 issue_pv(1, j);
-                umma_commit(&sm.v_empty[s]);
+                umma_commit(&sm.v_empty[sv]);
                 if (more) {
                     issue_s(1, j + 1);
-                    umma_commit(&sm.k_empty[(j + 1) & 1]);
+                    umma_commit(&sm.k_empty[sk1]);
                 }
             }
             if (!ok) {
@@ -490,12 +510,12 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             if (j == num_kt - 1 && t == 0) {
                 // Zero V rows past pos_max: those keys may hold NaN (slots past n_b,
                 // or pages never loaded) and 0 * NaN would poison the PV sums.
-                ok = __all_sync(kFull, mbar_wait(&sm.v_full[j & 1], (j >> 1) & 1, abort_flag));
+                ok = __all_sync(kFull, mbar_wait(&sm.v_full[j % kVStages], (j / kVStages) & 1, abort_flag));
                 if (!ok)
                     break;
                 if (key0 + row > pos_max) {
                     for (int h = 0; h < 2; ++h) {
-                        uint4 *rz = reinterpret_cast<uint4 *>(sm.v[j & 1] + h * kPanel + row * 128);
+                        uint4 *rz = reinterpret_cast<uint4 *>(sm.v[j % kVStages] + h * kPanel + row * 128);
 #pragma unroll
                         for (int c16 = 0; c16 < 8; ++c16)
                             rz[c16] = make_uint4(0, 0, 0, 0);
