@@ -34,6 +34,8 @@
 #include <cfloat>
 #include <cmath>
 
+#include <type_traits>
+
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -368,59 +370,89 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
         if (lane == 0) {
             const uint32_t id_qk = idesc_bf16(kRows, kKeys, 0, 0);
             const uint32_t id_pv = idesc_bf16(kRows, kD, 0, 1);
-            auto issue_s = [&](int t, int j) {  // S_t = Q_t K_j^T
-                const int s = j % kKStages;
+            // The issuing lane shares its SM sub-partition with softmax warps, so
+            // every instruction it spends between MMAs can leave the tensor pipe
+            // idle.  All operand descriptors share one high word (stride, fixed
+            // bits, swizzle); their low words are computed here once and the
+            // issue loop below, unrolled over the ring stages, only selects them.
+            const uint32_t d_hi = (uint32_t)(desc_sw128(smem_addr(sm.q[0]), 16, 1024) >> 32);
+            uint32_t q_lo[kTiles][kD / 16], k_lo[kKStages][kD / 16], v_lo[kVStages][kKeys / 16];
 #pragma unroll
-                for (int k = 0; k < kD / 16; ++k) {
-                    const int atom = k >> 2, kin = k & 3;
-                    const uint64_t a = desc_sw128(smem_addr(sm.q[t] + atom * kPanel) + kin * 32, 16, 1024);
-                    const uint64_t bd = desc_sw128(smem_addr(sm.k[s] + atom * kPanel) + kin * 32, 16, 1024);
-                    umma_ss(tmem + t * kRows, a, bd, id_qk, k > 0);
-                }
+            for (int k = 0; k < kD / 16; ++k) {
+                const int off = (k >> 2) * kPanel + (k & 3) * 32;
+#pragma unroll
+                for (int t = 0; t < kTiles; ++t)
+                    q_lo[t][k] = (uint32_t)desc_sw128(smem_addr(sm.q[t] + off), 16, 1024);
+#pragma unroll
+                for (int st = 0; st < kKStages; ++st)
+                    k_lo[st][k] = (uint32_t)desc_sw128(smem_addr(sm.k[st] + off), 16, 1024);
+            }
+#pragma unroll
+            for (int k = 0; k < kKeys / 16; ++k)
+#pragma unroll
+                for (int st = 0; st < kVStages; ++st)
+                    v_lo[st][k] = (uint32_t)desc_sw128(smem_addr(sm.v[st] + k * 2048), kPanel, 1024);
+            auto desc = [&](uint32_t lo) { return ((uint64_t)d_hi << 32) | lo; };
+            auto issue_s = [&](int t, auto stage) {  // S_t = Q_t K^T from K stage `stage`
+                constexpr int st = decltype(stage)::value;
+#pragma unroll
+                for (int k = 0; k < kD / 16; ++k)
+                    umma_ss(tmem + t * kRows, desc(q_lo[t][k]), desc(k_lo[st][k]), id_qk, k > 0);
                 umma_commit(&sm.s_full[t]);
             };
-            auto issue_pv = [&](int t, int j) {  // O_t += P_t V_j, P_t from TMEM
-                const int s = j % kVStages;
+            auto issue_pv = [&](int t, bool first, auto stage) {  // O_t += P_t V, P_t from TMEM
+                constexpr int st = decltype(stage)::value;
 #pragma unroll
-                for (int k = 0; k < kKeys / 16; ++k) {  // keys 16k .. 16k+15 = P columns 8k ..
-                    const uint64_t bd = desc_sw128(smem_addr(sm.v[s]) + k * 2048, kPanel, 1024);
-                    umma_ts(tmem + 256 + t * kRows, tmem + t * kRows + 8 * k, bd, id_pv,
-                            (j > 0 || k > 0) ? 1u : 0u);
-                }
+                for (int k = 0; k < kKeys / 16; ++k)  // keys 16k .. 16k+15 = P columns 8k ..
+                    umma_ts(tmem + 256 + t * kRows, tmem + t * kRows + 8 * k, desc(v_lo[st][k]), id_pv,
+                            (!first || k > 0) ? 1u : 0u);
                 umma_commit(&sm.o_done[t]);
             };
+            using S0 = std::integral_constant<int, 0>;
+            using S1 = std::integral_constant<int, 1>;
+            using S2 = std::integral_constant<int, 2>;
+            static_assert(kKStages == 3 && kVStages == 2, "the issue loop is unrolled over 6 tiles");
             bool ok = mbar_wait(&sm.q_full, 0, abort_flag) && mbar_wait(&sm.k_full[0], 0, abort_flag);
             if (ok) {
                 tc_fence_after();
-                issue_s(0, 0);
-                issue_s(1, 0);
+                issue_s(0, S0{});
+                issue_s(1, S0{});
                 umma_commit(&sm.k_empty[0]);
             }
-            for (int j = 0; j < num_kt && ok; ++j) {
-                const int sv = j % kVStages;
-                const int sk1 = (j + 1) % kKStages;
+            // one key tile: V_j in V stage sv, K_{j+1} in K stage sk1
+            auto step = [&](int j, auto sv_c, auto sk1_c) {
+                constexpr int sv = decltype(sv_c)::value, sk1 = decltype(sk1_c)::value;
                 const bool more = j + 1 < num_kt;
                 // tile A: PV_A(j) once P_A(j) is in TMEM, then S_A(j+1) over it
                 ok = mbar_wait(&sm.p_full[0], j & 1, abort_flag) &&
                      mbar_wait(&sm.v_full[sv], (j / kVStages) & 1, abort_flag) &&
                      (!more || mbar_wait(&sm.k_full[sk1], ((j + 1) / kKStages) & 1, abort_flag));
                 if (!ok)
-                    break;
+                    return;
                 tc_fence_after();
-                issue_pv(0, j);
+                issue_pv(0, j == 0, sv_c);
                 if (more)
-                    issue_s(0, j + 1);
+                    issue_s(0, sk1_c);
                 // tile B likewise; then V_j and K_{j+1} are no longer needed
                 ok = mbar_wait(&sm.p_full[1], j & 1, abort_flag);
                 if (!ok)
-                    break;
+                    return;
                 tc_fence_after();
-                issue_pv(1, j);
+                issue_pv(1, j == 0, sv_c);
                 umma_commit(&sm.v_empty[sv]);
                 if (more) {
-                    issue_s(1, j + 1);
+                    issue_s(1, sk1_c);
                     umma_commit(&sm.k_empty[sk1]);
                 }
+            };
+            for (int j0 = 0; j0 < num_kt && ok; j0 += 6) {
+                // (j mod 2, (j + 1) mod 3) for j = j0 .. j0 + 5, j0 a multiple of 6
+                step(j0, S0{}, S1{});
+                if (ok && j0 + 1 < num_kt) step(j0 + 1, S1{}, S2{});
+                if (ok && j0 + 2 < num_kt) step(j0 + 2, S0{}, S0{});
+                if (ok && j0 + 3 < num_kt) step(j0 + 3, S1{}, S1{});
+                if (ok && j0 + 4 < num_kt) step(j0 + 4, S0{}, S2{});
+                if (ok && j0 + 5 < num_kt) step(j0 + 5, S1{}, S0{});
             }
             if (!ok) {
                 *abort_flag = 1;
