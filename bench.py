@@ -400,6 +400,74 @@ def bench_staging(device, reps, layers=2, batch=None):
     return res
 
 
+def bench_host_staging(device, reps, layers=2, batch=8):
+    """Prefix staging to and from page-locked host memory: the copy kernel reads
+    the pool and writes the rows straight over the CPU-GPU link (and the inverse
+    for the load).  The link's own figure is a cudaMemcpyAsync of the same bytes
+    between a device buffer and the same pinned buffer."""
+    job = make_staging_job(STAGING, batch=batch)
+    k_layers = [torch.empty((job.num_pages, 8, 16, 128), dtype=torch.bfloat16, device=device)
+                for _ in range(layers)]
+    v_layers = [torch.empty_like(k_layers[0]) for _ in range(layers)]
+    for l in range(layers):
+        fill_layer_pool(k_layers[l], v_layers[l], STAGING.seed, l)
+    pool = cadkv.KVPool(k_layers, v_layers)
+    lens = job.context_lens
+    size = cadkv.staged_size(lens, 0, layers, 8, 128)
+    host = torch.empty(size, dtype=torch.bfloat16, pin_memory=True)
+    dev = torch.empty(size, dtype=torch.bfloat16, device=device)
+    bt = torch.from_numpy(job.block_table).to(device)
+    cl = torch.from_numpy(lens).to(device)
+    ws = torch.empty(cadkv.kv_prefix_stage_workspace_size(len(lens)), dtype=torch.uint8,
+                     device=device)
+    stream = torch.cuda.current_stream(device)
+
+    def timed(fn):
+        for _ in range(2):
+            fn()
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(reps)]
+        for e0, e1 in ev:
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        return statistics.mean(e0.elapsed_time(e1) for e0, e1 in ev)
+
+    to_host_ms = timed(lambda: cadkv.kv_prefix_stage(pool, bt, cl, 0, layers, host,
+                                                     workspace=ws, stream=stream))
+    to_host_status = cadkv.kv_prefix_stage_status(ws)
+    cadkv.kv_prefix_stage(pool, bt, cl, 0, layers, dev, workspace=ws, stream=stream)
+    torch.cuda.synchronize()
+    exact = bool(torch.equal(host.to(device, non_blocking=False).view(torch.int16),
+                             dev.view(torch.int16)))
+    from_host_ms = timed(lambda: cadkv.kv_prefix_load(pool, bt, cl, 0, layers, host,
+                                                      workspace=ws, stream=stream))
+    from_host_status = cadkv.kv_prefix_stage_status(ws)
+    d2h_ms = timed(lambda: host.copy_(dev, non_blocking=True))
+    h2d_ms = timed(lambda: dev.copy_(host, non_blocking=True))
+    nbytes = size * 2
+
+    def gbs(ms):
+        return round(nbytes / (ms * 1e-3) / 1e9, 1)
+
+    res = {"workload": f"{STAGING.name}: first {len(lens)} trajectories, {layers} of 48 layers, "
+                       "rows in page-locked host memory",
+           "bytes_over_link_per_call": nbytes,
+           "to_host": {"gbps": gbs(to_host_ms), "ms_per_call": round(to_host_ms, 3),
+                       "status": to_host_status, "bit_exact_vs_device_staging": exact,
+                       "frac_of_memcpy_d2h": round(d2h_ms / to_host_ms, 4)},
+           "from_host": {"gbps": gbs(from_host_ms), "ms_per_call": round(from_host_ms, 3),
+                         "status": from_host_status,
+                         "frac_of_memcpy_h2d": round(h2d_ms / from_host_ms, 4)},
+           "link_reference": {"memcpy_d2h_gbps": gbs(d2h_ms), "memcpy_h2d_gbps": gbs(h2d_ms),
+                              "note": "cudaMemcpyAsync of the same bytes, contiguous, no gather"}}
+    del host, dev, k_layers, v_layers, pool
+    torch.cuda.empty_cache()
+    return res
+
+
 def read_probe(buf, reps=10):
     """Pure-read bandwidth (GB/s) of ``buf`` with the library's read probe."""
     sink = torch.zeros(1, dtype=torch.int64, device=buf.device)
@@ -570,6 +638,7 @@ def main():
     if args.workload == "staging":
         res = bench_staging(device, reps=args.steps, layers=args.staging_layers,
                             batch=args.staging_batch)
+        res["host"] = bench_host_staging(device, reps=args.steps)
         if rank == 0:
             print(json.dumps(res), flush=True)
         return
@@ -674,6 +743,7 @@ def main():
     torch.cuda.empty_cache()
     if rank == 0 and not args.no_extras:
         line["staging"] = bench_staging(device, reps=10, layers=args.staging_layers)
+        line["staging"]["host"] = bench_host_staging(device, reps=5)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -255,13 +255,20 @@ size_t kv_prefix_stage_workspace_size(int batch);
 
 /*
  * Gather the first n_b tokens of layers [layer_begin, layer_end) of every
- * trajectory b from the pool into contiguous rows:
+ * trajectory b from the pool into contiguous rows (Sec. 5, late-bound KV
+ * preparation: the departing trajectory's prefix is snapshotted):
  *   dst[off_b + (((l - layer_begin)*2 + kv)*Hkv + h)*n_b*D + t*D + d]
  *       = (kv == 0 ? K : V)_l[block_table[b][t/16]][h][t%16][d]
  * off_b = dst_offsets[b] (device int64 [batch], elements, multiples of 8) or,
  * when dst_offsets is NULL, (layer_end - layer_begin)*2*Hkv*D*sum_{b'<b} n_b'.
  * A bit-exact copy: every bf16 pattern, NaN payloads included, is preserved.
  * Elements of dst outside the rows are not written.
+ * dst (host or device): device memory, or page-locked host memory the device
+ * can address (cudaHostAlloc / cudaHostRegister; a pinned torch tensor).  With
+ * host memory the kernel writes the rows straight over the CPU-GPU link
+ * (NVLink-C2C on Grace systems), so a snapshot reaches host memory in one pass
+ * with no device-side staging buffer.  Pageable host memory: CADKV_ERR_INVALID.
+ * The caller keeps dst alive until the stream reaches the call.
  */
 int kv_prefix_stage(const cadkv_pool *pool, const int32_t *block_table, int max_pages,
                     const int32_t *context_lens, int batch, int layer_begin,
@@ -272,6 +279,8 @@ int kv_prefix_stage(const cadkv_pool *pool, const int32_t *block_table, int max_
  * Inverse of kv_prefix_stage: write staged rows `src` (same layout and
  * offsets) into the pool pages named by block_table.  Slots of a last page
  * past n_b are not written.  Pages named twice give an unspecified result.
+ * src may be page-locked host memory, as dst of kv_prefix_stage: a prefix
+ * kept in host memory is loaded into a destination pool in one pass.
  */
 int kv_prefix_load(const cadkv_pool *pool, const int32_t *block_table, int max_pages,
                    const int32_t *context_lens, int batch, int layer_begin,

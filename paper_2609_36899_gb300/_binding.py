@@ -373,7 +373,11 @@ def _stage_common(fn, name, pool: KVPool, block_table, context_lens, layer_begin
     dev = pool.device
     _need(block_table, "block_table", torch.int32, 2, dev)
     _need(context_lens, "context_lens", torch.int32, 1, dev)
-    _need(rows, "rows", torch.bfloat16, None, dev)
+    if rows.is_cuda:
+        _need(rows, "rows", torch.bfloat16, None, dev)
+    else:  # page-locked host rows: the kernel reads or writes them over the link
+        if rows.dtype != torch.bfloat16 or not rows.is_contiguous() or not rows.is_pinned():
+            raise ValueError("host rows must be a contiguous, pinned bfloat16 tensor")
     if offsets is not None:
         _need(offsets, "offsets", torch.int64, 1, dev)
     batch = context_lens.shape[0]
@@ -391,7 +395,8 @@ def _stage_common(fn, name, pool: KVPool, block_table, context_lens, layer_begin
 
 def kv_prefix_stage(pool: KVPool, block_table, context_lens, layer_begin: int,
                     layer_end: int, dst, dst_offsets=None, workspace=None, stream=None):
-    """Gather each trajectory's prefix of layers [layer_begin, layer_end) into ``dst``."""
+    """Gather each trajectory's prefix of layers [layer_begin, layer_end) into ``dst``
+    (a CUDA tensor, or a pinned CPU tensor written directly over the CPU-GPU link)."""
     return _stage_common(library().kv_prefix_stage, "kv_prefix_stage", pool, block_table,
                          context_lens, layer_begin, layer_end, dst, dst_offsets, workspace,
                          stream)
@@ -399,7 +404,8 @@ def kv_prefix_stage(pool: KVPool, block_table, context_lens, layer_begin: int,
 
 def kv_prefix_load(pool: KVPool, block_table, context_lens, layer_begin: int,
                    layer_end: int, src, src_offsets=None, workspace=None, stream=None):
-    """Write staged rows ``src`` into the pool pages named by ``block_table``."""
+    """Write staged rows ``src`` (CUDA, or pinned CPU) into the pool pages named by
+    ``block_table``."""
     return _stage_common(library().kv_prefix_load, "kv_prefix_load", pool, block_table,
                          context_lens, layer_begin, layer_end, src, src_offsets, workspace,
                          stream)

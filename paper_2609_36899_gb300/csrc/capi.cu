@@ -306,6 +306,20 @@ int stage_impl(const cadkv_pool *pool, const int32_t *block_table, int max_pages
     const StageWorkspaceLayout L = stage_workspace_layout(batch);
     if (!workspace || !aligned(workspace, kWorkspaceAlign) || workspace_bytes < L.total)
         return CADKV_ERR_WORKSPACE;
+    // The staged rows may be device memory or page-locked host memory that the
+    // device can address (then the copy kernel reads or writes host memory
+    // directly over the CPU-GPU link); pageable host memory is refused.
+    cudaPointerAttributes attr{};
+    if (cudaPointerGetAttributes(&attr, rows) != cudaSuccess) {
+        cudaGetLastError();
+        return CADKV_ERR_INVALID;
+    }
+    if (attr.type == cudaMemoryTypeUnregistered ||
+        (attr.type == cudaMemoryTypeHost && attr.devicePointer == nullptr))
+        return CADKV_ERR_INVALID;
+    const void *dev_rows = attr.type == cudaMemoryTypeHost ? attr.devicePointer : rows;
+    if (!aligned(dev_rows, 16))
+        return CADKV_ERR_INVALID;
     const int sms = device_sms();
     if (sms < 0)
         return sms;
@@ -315,7 +329,7 @@ int stage_impl(const cadkv_pool *pool, const int32_t *block_table, int max_pages
     p.layer_v = pool->dev_layer_ptrs + pool->num_layers;
     p.block_table = block_table;
     p.context_lens = context_lens;
-    p.rows = const_cast<void *>(rows);
+    p.rows = const_cast<void *>(dev_rows);
     p.row_offsets = reinterpret_cast<const long long *>(offsets);
     p.hdr = reinterpret_cast<WorkspaceHeader *>(ws);
     p.page_prefix = reinterpret_cast<long long *>(ws + L.page_prefix);

@@ -134,6 +134,67 @@ def test_load_round_trip():
     assert torch.equal(again.view(torch.int16), staged.view(torch.int16))
 
 
+def test_stage_to_pinned_host_bit_exact():
+    """Staging straight into page-locked host memory (the copy kernel writes the
+    rows over the CPU-GPU link) gives the oracle's bytes and leaves the bytes
+    after the rows untouched."""
+    lens, table, kp, vp = make_case([1, 15, 16, 17, 40, 0, 333, 1000], 2, 8, 128, seed=26)
+    pool, _, _ = to_pool(kp, vp)
+    size = cadkv.staged_size(lens, 0, 2, 8, 128)
+    dst = torch.empty(size + 64, dtype=torch.bfloat16, pin_memory=True)
+    dst.view(torch.int16).fill_(0x1234)
+    ws = cadkv.kv_prefix_stage(pool, torch.from_numpy(table).cuda(),
+                               torch.from_numpy(lens).cuda(), 0, 2, dst)
+    assert cadkv.kv_prefix_stage_status(ws) == 0  # synchronises the stream
+    got = bf16_bits(dst)
+    np.testing.assert_array_equal(got[:size], oracle_stage(kp, vp, table, lens, 0, 2))
+    assert np.all(got[size:] == 0x1234)
+
+
+def test_load_from_pinned_host_round_trip():
+    """Rows kept in page-locked host memory load into a fresh pool (another page
+    table) exactly as the oracle's load writes them."""
+    lens, table, kp, vp = make_case([21, 64, 2, 0, 100], 2, 2, 128, seed=27)
+    pool, _, _ = to_pool(kp, vp)
+    lens_d = torch.from_numpy(lens).cuda()
+    staged = torch.empty(cadkv.staged_size(lens, 0, 2, 2, 128), dtype=torch.bfloat16,
+                         pin_memory=True)
+    ws = cadkv.kv_prefix_stage(pool, torch.from_numpy(table).cuda(), lens_d, 0, 2, staged)
+    assert cadkv.kv_prefix_stage_status(ws) == 0
+    rng = np.random.Generator(np.random.PCG64(28))
+    pages = int((-(-lens.astype(np.int64) // 16)).sum())
+    table2, n2 = scatter_block_table(lens, 16, table.shape[1], pages + 4, rng)
+    k2 = torch.zeros((2, n2, 2, 16, 128), dtype=torch.bfloat16)
+    pool2, k2_layers, v2_layers = to_pool(k2, torch.zeros_like(k2))
+    ws = cadkv.kv_prefix_load(pool2, torch.from_numpy(table2).cuda(), lens_d, 0, 2, staged)
+    assert cadkv.kv_prefix_stage_status(ws) == 0
+    ref_k = np.zeros((2, n2, 2, 16, 128), dtype=np.uint16)
+    ref_v = np.zeros_like(ref_k)
+    oracle.prefix_load(ref_k, ref_v, table2, lens, 0, 2, bf16_bits(staged))
+    np.testing.assert_array_equal(np.stack([bf16_bits(t) for t in k2_layers]), ref_k)
+    np.testing.assert_array_equal(np.stack([bf16_bits(t) for t in v2_layers]), ref_v)
+
+
+def test_stage_refuses_pageable_host_rows():
+    """Host rows that are not page-locked are refused before anything launches,
+    by the binding and by the C ABI itself."""
+    import ctypes
+    lens, table, kp, vp = make_case([20], 1, 1, 64, seed=29)
+    pool, _, _ = to_pool(kp, vp)
+    bt = torch.from_numpy(table).cuda()
+    cl = torch.from_numpy(lens).cuda()
+    dst = torch.zeros(cadkv.staged_size(lens, 0, 1, 1, 64) + 64, dtype=torch.bfloat16)
+    with pytest.raises(ValueError):
+        cadkv.kv_prefix_stage(pool, bt, cl, 0, 1, dst)
+    ws = torch.empty(cadkv.kv_prefix_stage_workspace_size(1), dtype=torch.uint8, device="cuda")
+    P = ctypes.c_void_p
+    rc = cadkv.library().kv_prefix_stage(pool.handle, P(bt.data_ptr()), bt.shape[1],
+                                         P(cl.data_ptr()), 1, 0, 1, P(dst.data_ptr()), None,
+                                         P(ws.data_ptr()), ws.numel(), None)
+    assert rc == STATUS["CADKV_ERR_INVALID"]
+    assert torch.count_nonzero(dst.view(torch.int16)) == 0
+
+
 def test_full_size_staging_sampled():
     """All 64 trajectories of the staging workload (lengths 8K..64K tokens,
     8 KV heads, D = 128) for two layers; every staged row of four sampled
