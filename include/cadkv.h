@@ -232,7 +232,8 @@ size_t prefill_attention_workspace_size(int batch);
  * to keys 0 .. p:  out = softmax_t<=p(q . K_t / sqrt(D)) V,  lse = ln sum exp.
  * Runs on the tcgen05 tensor cores (accumulators in TMEM), one CTA per
  * (trajectory, KV head, tile of 128 (query token, head) rows).
- * Supported: head_dim 128, page_size 16, G = Hq / Hkv in {1, 2, 4, 8}.
+ * Supported: head_dim 128, page_size 16, G = Hq / Hkv in 1..8 (the Qwen3
+ * models of Sec. 6 have G = 4, 5 and 8).
  * A trajectory with C_b > n_b or n_b out of range is skipped (its rows are
  * not written) and CADKV_ERR_SHAPE lands in the status word.
  */

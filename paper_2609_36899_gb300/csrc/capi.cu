@@ -573,8 +573,7 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
         num_pages <= 0 || num_q_heads % num_kv_heads != 0)
         return CADKV_ERR_SHAPE;
     const int group = num_q_heads / num_kv_heads;
-    if (head_dim != 128 || page_size != kPageSize ||
-        (group != 1 && group != 2 && group != 4 && group != 8))
+    if (head_dim != 128 || page_size != kPageSize || group > kMaxGroup)
         return CADKV_ERR_UNSUPPORTED;
     if ((long long)num_pages * num_kv_heads * kPageSize > INT32_MAX ||
         (long long)max_pages * kPageSize > INT32_MAX)
@@ -593,7 +592,8 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
     EncodeTiledFn fn = encode_tiled_fn();
     if (!fn)
         return CADKV_ERR_CUDA;
-    // Q viewed as {D, Hq, T}: box {64, G, 128/G} = 128 rows (token-major, head-minor)
+    // Q viewed as {D, Hq, T}: box {64, G, floor(128/G)} = up to 128 rows (token-major,
+    // head-minor)
     CUtensorMap qmap, kmap, vmap;
     {
         const cuuint64_t dims[3] = {(cuuint64_t)head_dim, (cuuint64_t)num_q_heads,
@@ -631,10 +631,9 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
     p.max_pages = max_pages;
     p.num_pages = num_pages;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
-    // upper bound on work items: sum_b ceil(C_b G / R) <= T G / R + B, R rows per item
-    const long long rows = prefill_rows_per_item();
-    const long long grid =
-        (long long)num_kv_heads * (batch + ((long long)total_q * group + rows - 1) / rows);
+    // upper bound on work items: sum_b ceil(C_b / U) <= T / U + B, U tokens per item
+    const long long tpi = prefill_tokens_per_item(group);
+    const long long grid = (long long)num_kv_heads * (batch + ((long long)total_q + tpi - 1) / tpi);
     if (grid > INT32_MAX)
         return CADKV_ERR_UNSUPPORTED;
     return launch_prefill(p, qmap, kmap, vmap, (int)grid, reinterpret_cast<cudaStream_t>(stream)) ==

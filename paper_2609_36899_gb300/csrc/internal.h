@@ -102,7 +102,9 @@ struct PrefillParams {
 };
 
 size_t prefill_smem_bytes();
-int prefill_rows_per_item();  // (query token, head) rows one prefill CTA handles
+// query tokens one prefill CTA handles for head group `group` (two tiles of
+// floor(128 / group) tokens, all heads of the group)
+__host__ __device__ long long prefill_tokens_per_item(int group);
 cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, const CUtensorMap &kmap,
                            const CUtensorMap &vmap, int grid, cudaStream_t stream);
 

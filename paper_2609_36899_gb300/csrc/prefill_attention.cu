@@ -176,7 +176,8 @@ __global__ void __launch_bounds__(1024, 1) prefill_plan_kernel(const PrefillPara
                 n > p.max_pages * kPageSize) {
                 record_status(&p.hdr->status, CADKV_ERR_SHAPE);
             } else {
-                items = (long long)p.num_kv_heads * ((c * p.group + kItemRows - 1) / kItemRows);
+                const long long tpi = prefill_tokens_per_item(p.group);
+                items = (long long)p.num_kv_heads * ((c + tpi - 1) / tpi);
             }
         }
         long long v = items;
@@ -241,11 +242,14 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
     }
     const int b = lo;
     const int G = p.group;
+    // a tile holds floor(128 / G) whole tokens (all G heads of each); for G that
+    // does not divide 128 the last 128 mod G rows are padding, never written out
     const int tokens_per_tile = kRows / G;
+    const int rows_used = tokens_per_tile * G;
     const long long q0 = p.q_offsets[b];
     const int chunk = (int)(p.q_offsets[b + 1] - q0);
     const int n = p.context_lens[b];
-    const int qblocks = (chunk * G + kItemRows - 1) / kItemRows;
+    const int qblocks = (chunk + kTiles * tokens_per_tile - 1) / (kTiles * tokens_per_tile);
     const int local = (int)(item - p.item_prefix[b]);
     const int g = local / qblocks;
     const int qt = qblocks - 1 - local % qblocks;  // heaviest blocks first
@@ -275,6 +279,16 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
         sm.abort = 0;
         fence_mbarrier_init();
     }
+    if (rows_used < kRows) {
+        // padding rows of both Q tiles: zero them so the MMAs read finite values
+        // (the Q copies never write them)
+        const int pad = kRows - rows_used;
+        for (int i = tid; i < kTiles * 2 * pad * 8; i += kPrefillThreads) {
+            const int t = i / (2 * pad * 8), h = (i / (pad * 8)) % 2, r = rows_used + (i / 8) % pad;
+            reinterpret_cast<uint4 *>(sm.q[t] + h * kPanel + r * 128)[i % 8] = make_uint4(0, 0, 0, 0);
+        }
+        fence_proxy_async_smem();
+    }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
                          smem_addr(&sm.tmem_base))
@@ -298,7 +312,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             prefetch_tensor_map(&qmap);
             prefetch_tensor_map(&kmap);
             prefetch_tensor_map(&vmap);
-            mbar_arrive_expect_tx(&sm.q_full, kTiles * kTileBytes);
+            mbar_arrive_expect_tx(&sm.q_full, kTiles * 2 * rows_used * 128);
             for (int t = 0; t < kTiles; ++t) {
                 const int qy = (int)(q0 + i0 + t * tokens_per_tile);
                 for (int h = 0; h < 2; ++h)
@@ -472,7 +486,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
         const uint32_t s_col = tmem + lane_base + t * kRows;
         const uint32_t o_col = tmem + lane_base + 256 + t * kRows;
         const int token = t * tokens_per_tile + row / G, head = row % G;
-        const bool row_valid = token < valid_tokens;
+        const bool row_valid = row < rows_used && token < valid_tokens;
         const int pos_row = row_valid ? chunk_start + i0 + token : pos_max;
         const int pos_min = chunk_start + i0 + t * tokens_per_tile;  // first row of the tile
         const float scale = p.scale_log2;
@@ -605,7 +619,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
 
 size_t prefill_smem_bytes() { return sizeof(PrefillSmem) + 1024; }
 
-int prefill_rows_per_item() { return kItemRows; }
+__host__ __device__ long long prefill_tokens_per_item(int group) { return (long long)kTiles * (kRows / group); }
 
 cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, const CUtensorMap &kmap,
                            const CUtensorMap &vmap, int grid, cudaStream_t stream)

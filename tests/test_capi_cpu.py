@@ -119,7 +119,7 @@ def test_prefill_rejects_on_host(lib):
                                      args["hq"], args["hkv"], args["d"], args["page"],
                                      args["num_pages"], args["max_pages"], a, 1 << 20, None)
     assert call(d=64) == STATUS["CADKV_ERR_UNSUPPORTED"]
-    assert call(hq=6, hkv=2) == STATUS["CADKV_ERR_UNSUPPORTED"]      # G = 3
+    assert call(hq=18, hkv=2) == STATUS["CADKV_ERR_UNSUPPORTED"]     # G = 9 > 8
     assert call(hq=6, hkv=4) == STATUS["CADKV_ERR_SHAPE"]
     assert call(q=None) == STATUS["CADKV_ERR_INVALID"]
     assert call(offs=P((1 << 12) + 4)) == STATUS["CADKV_ERR_INVALID"]

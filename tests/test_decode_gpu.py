@@ -64,7 +64,8 @@ def test_full_size_sampled(w):
     torch.cuda.empty_cache()
 
 
-@pytest.mark.parametrize("g,d", [(1, 64), (2, 128), (4, 64), (8, 128), (8, 64), (3, 128)])
+@pytest.mark.parametrize("g,d", [(1, 64), (2, 128), (4, 64), (8, 128), (8, 64), (3, 128),
+                                 (5, 128)])
 def test_edge_lengths(g, d):
     lens = [0, 1, 2, 15, 16, 17, 31, 32, 33, 255, 256, 257, 1000]
     hkv = 2

@@ -41,7 +41,7 @@ def _oracle(batch, offs, q):
                                     batch.context_lens)
 
 
-@pytest.mark.parametrize("g", [1, 2, 4, 8])
+@pytest.mark.parametrize("g", [1, 2, 3, 4, 5, 6, 7, 8])
 def test_prefill_small(g):
     lens, chunks = [40, 300, 17, 130], [40, 5, 17, 129]
     batch, offs, q = _case(lens, chunks, 2 * g, 2, seed=400 + g)
@@ -67,6 +67,17 @@ def test_prefill_qwen_shape():
     out, lse, ws = _run(batch, offs, q)
     ref, ref_lse = _oracle(batch, offs, q)
     assert_close(out, lse, ref, ref_lse, "prefill 32/8")
+
+
+def test_prefill_qwen14b_shape():
+    """40 query / 8 KV heads (G = 5: a tile holds 25 tokens, 125 rows + 3 padding
+    rows), chunks spanning several query tiles and items, ragged tails."""
+    lens, chunks = [3000, 1200, 60], [200, 77, 60]
+    batch, offs, q = _case(lens, chunks, 40, 8, seed=425)
+    out, lse, ws = _run(batch, offs, q)
+    assert cadkv.prefill_attention_status(ws) == 0
+    ref, ref_lse = _oracle(batch, offs, q)
+    assert_close(out, lse, ref, ref_lse, "prefill 40/8")
 
 
 def test_prefill_chunk_of_one_matches_decode():
