@@ -39,9 +39,10 @@ sys.path.insert(0, ROOT)
 
 import paper_2609_36899_gb300 as cadkv  # noqa: E402
 from paper_2609_36899_gb300 import build as pkg_build  # noqa: E402
-from paper_2609_36899_gb300.workloads import (DECODE_WORKLOADS, STAGING, bf16_bits,  # noqa: E402
-                                              fill_layer_pool, landscape_workload,
-                                              make_decode_batch, make_staging_job)
+from paper_2609_36899_gb300.workloads import (DECODE_WORKLOADS, PREFILL, STAGING,  # noqa: E402
+                                              bf16_bits, fill_layer_pool, landscape_workload,
+                                              make_decode_batch, make_prefill_job,
+                                              make_staging_job)
 
 METRIC = "decode-attention achieved HBM GB/s (% of 8 TB/s) and decode steps/s per batch"
 NOMINAL_HBM_GBS = 8000.0
@@ -519,16 +520,12 @@ def bench_landscape(device, steps, warmup, batches=(8, 32, 128, 512),
     return cells
 
 
-def bench_prefill(device, steps, warmup, batch=8, context=16384, chunk=512, hq=32, hkv=8):
-    """Chunked re-prefill: each of `batch` trajectories recomputes attention for
-    its last `chunk` tokens over a `context`-token paged KV (32/8 heads, D=128)."""
-    from paper_2609_36899_gb300.workloads import DecodeWorkload
-    w = DecodeWorkload("prefill", batch, hq, hkv, 128, "fixed", tuple([context] * batch),
-                       context, 20267)
-    b = make_decode_batch(w, device=device)
-    offs = torch.arange(0, (batch + 1) * chunk, chunk, dtype=torch.int64, device=device)
-    g = torch.Generator(device=device).manual_seed(20268)
-    q = torch.randn((batch * chunk, hq, 128), generator=g, device=device).to(torch.bfloat16)
+def bench_prefill(device, steps, warmup):
+    """Chunked re-prefill: each of 8 trajectories recomputes attention for its
+    last 512 tokens over a 16,384-token paged KV (32/8 heads, D=128)."""
+    w = PREFILL
+    batch, context, chunk, hq, hkv = w.batch, w.context, w.chunk, w.num_q_heads, w.num_kv_heads
+    b, offs, q = make_prefill_job(w, device)
     bt = torch.from_numpy(b.block_table).to(device)
     cl = torch.from_numpy(b.context_lens).to(device)
     out = torch.empty_like(q)

@@ -79,6 +79,23 @@ DECODE_WORKLOADS = {"tiny": TINY, "paced": PACED, "long_tail": LONG_TAIL,
                     "mixed": MIXED}
 
 
+@dataclass(frozen=True)
+class PrefillWorkload:
+    """Shape of one chunked re-prefill job: each of `batch` trajectories of
+    `context` tokens recomputes attention for its last `chunk` tokens."""
+    name: str
+    batch: int
+    context: int
+    chunk: int
+    num_q_heads: int
+    num_kv_heads: int
+    head_dim: int
+    seed: int
+
+
+PREFILL = PrefillWorkload("chunked prefill", 8, 16384, 512, 32, 8, 128, 20267)
+
+
 def landscape_workload(batch: int, mean_len: int, seed: int = 20266) -> DecodeWorkload:
     """One cell of the decode-throughput landscape over (B, mean context C):
     lengths uniform in [C/2, 3C/2], 32 query / 8 KV heads, head_dim 128 (the
@@ -186,6 +203,19 @@ def make_decode_batch(w: DecodeWorkload, device="cpu", seed: int | None = None,
     k = _randn_bf16_chunked(kv_shape, gen, device, w.k_scale)
     v = _randn_bf16_chunked(kv_shape, gen, device)
     return DecodeBatch(w, lens, table, q, k, v)
+
+
+def make_prefill_job(w: PrefillWorkload, device="cpu"):
+    """The paged pool (fixed lengths, scattered pages), the chunk offsets
+    (int64 [batch + 1]) and the queries (bf16 [batch * chunk, Hq, D]) of ``w``."""
+    dw = DecodeWorkload(w.name, w.batch, w.num_q_heads, w.num_kv_heads, w.head_dim, "fixed",
+                        tuple([w.context] * w.batch), w.context, w.seed)
+    b = make_decode_batch(dw, device=device)
+    offs = torch.arange(0, (w.batch + 1) * w.chunk, w.chunk, dtype=torch.int64, device=device)
+    g = torch.Generator(device=device).manual_seed(w.seed + 1)
+    q = torch.randn((w.batch * w.chunk, w.num_q_heads, w.head_dim), generator=g,
+                    device=device).to(torch.bfloat16)
+    return b, offs, q
 
 
 @dataclass
