@@ -284,6 +284,35 @@ int read_status(const void *workspace, cudaStream_t stream)
     return status;
 }
 
+// Persistent CTAs of the prefill kernel: one per SM of the current device (an
+// upper bound when no device answers, so that a size query never comes short).
+int prefill_ctas()
+{
+    const int sms = device_sms();
+    return sms > 0 ? sms : 256;
+}
+
+struct PrefillWorkspaceLayout {
+    size_t item_prefix, merge_counter, partial_lambda, partial_o, total;
+};
+
+PrefillWorkspaceLayout prefill_workspace_layout(int batch, int ctas)
+{
+    PrefillWorkspaceLayout L{};
+    size_t off = align_up_host(sizeof(WorkspaceHeader), kWorkspaceAlign);
+    L.item_prefix = off;
+    off += align_up_host((size_t)(batch + 1) * sizeof(long long), kWorkspaceAlign);
+    L.merge_counter = off;
+    off += align_up_host((size_t)ctas * sizeof(int), kWorkspaceAlign);
+    const size_t slots = (size_t)2 * ctas * 256;
+    L.partial_lambda = off;
+    off += align_up_host(slots * sizeof(float), kWorkspaceAlign);
+    L.partial_o = off;
+    off += align_up_host(slots * 128 * sizeof(float), kWorkspaceAlign);
+    L.total = off;
+    return L;
+}
+
 int stage_impl(const cadkv_pool *pool, const int32_t *block_table, int max_pages,
                const int32_t *context_lens, int batch, int layer_begin, int layer_end,
                const void *rows, const int64_t *offsets, void *workspace,
@@ -558,8 +587,7 @@ size_t prefill_attention_workspace_size(int batch)
 {
     if (batch < 0)
         return 0;
-    return align_up_host(sizeof(WorkspaceHeader), kWorkspaceAlign) +
-           align_up_host((size_t)(batch + 1) * sizeof(long long), kWorkspaceAlign);
+    return prefill_workspace_layout(batch, prefill_ctas()).total;
 }
 
 int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pages,
@@ -613,6 +641,8 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
         encode_pages_map(&vmap, v_pages, num_pages, num_kv_heads, head_dim, false, &whole) !=
             CADKV_OK)
         return CADKV_ERR_CUDA;
+    const int ctas = prefill_ctas();
+    const PrefillWorkspaceLayout L = prefill_workspace_layout(batch, ctas);
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     PrefillParams p{};
     p.q_offsets = reinterpret_cast<const long long *>(q_offsets);
@@ -621,8 +651,11 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
     p.out = static_cast<__nv_bfloat16 *>(out);
     p.lse = lse;
     p.hdr = reinterpret_cast<WorkspaceHeader *>(ws);
-    p.item_prefix = reinterpret_cast<long long *>(ws + align_up_host(sizeof(WorkspaceHeader),
-                                                                      kWorkspaceAlign));
+    p.item_prefix = reinterpret_cast<long long *>(ws + L.item_prefix);
+    p.merge_counter = reinterpret_cast<int *>(ws + L.merge_counter);
+    p.partial_lambda = reinterpret_cast<float *>(ws + L.partial_lambda);
+    p.partial_o = reinterpret_cast<float *>(ws + L.partial_o);
+    p.num_ctas = ctas;
     p.total_q = total_q;
     p.batch = batch;
     p.num_q_heads = num_q_heads;
@@ -631,12 +664,7 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
     p.max_pages = max_pages;
     p.num_pages = num_pages;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
-    // upper bound on work items: sum_b ceil(C_b / U) <= T / U + B, U tokens per item
-    const long long tpi = prefill_tokens_per_item(group);
-    const long long grid = (long long)num_kv_heads * (batch + ((long long)total_q + tpi - 1) / tpi);
-    if (grid > INT32_MAX)
-        return CADKV_ERR_UNSUPPORTED;
-    return launch_prefill(p, qmap, kmap, vmap, (int)grid, reinterpret_cast<cudaStream_t>(stream)) ==
+    return launch_prefill(p, qmap, kmap, vmap, reinterpret_cast<cudaStream_t>(stream)) ==
                    cudaSuccess
                ? CADKV_OK
                : CADKV_ERR_CUDA;

@@ -26,8 +26,11 @@ struct alignas(64) WorkspaceHeader {
     int slice_counter;     // next work slice to hand out
     int num_slices;        // T: slices of the flattened work sequence
     int pad0;
-    long long total_work;  // W: page-heads (decode) or copy units (staging)
-    long long pad1[5];
+    long long total_work;  // W: page-heads (decode), copy units (staging), work units (prefill)
+    long long total_items; // prefill: work items
+    long long dp_items;    // prefill: items run whole (the rest are split)
+    long long pieces;      // prefill: pieces per split item
+    long long pad1[2];
 };
 
 // Byte offsets of the decode-attention workspace regions.
@@ -94,19 +97,19 @@ struct PrefillParams {
     const int *block_table;
     __nv_bfloat16 *out;          // [T][Hq][D]
     float *lse;                  // [T][Hq], nullable
-    WorkspaceHeader *hdr;
-    long long *item_prefix;      // [batch + 1]
+    WorkspaceHeader *hdr;        // total_work = work units; slice_counter = next unit
+    long long *item_prefix;      // [batch + 1] work items of trajectories before b
+    int *merge_counter;          // [num_ctas] pieces done of split item i
+    float *partial_lambda;       // [2 * num_ctas][256] log2-lse of a piece's rows
+    float *partial_o;            // [2 * num_ctas][256][128] O / l of a piece's rows
     long long total_q;           // rows of q / out; offsets beyond it are rejected
-    int batch, num_q_heads, num_kv_heads, group, max_pages, num_pages;
+    int batch, num_q_heads, num_kv_heads, group, max_pages, num_pages, num_ctas;
     float scale_log2;
 };
 
 size_t prefill_smem_bytes();
-// query tokens one prefill CTA handles for head group `group` (two tiles of
-// floor(128 / group) tokens, all heads of the group)
-__host__ __device__ long long prefill_tokens_per_item(int group);
 cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, const CUtensorMap &kmap,
-                           const CUtensorMap &vmap, int grid, cudaStream_t stream);
+                           const CUtensorMap &vmap, cudaStream_t stream);
 
 // ---------------------------------------------------------------- staging
 

@@ -6,16 +6,28 @@
 // trajectory's last C_b tokens attend causally over its paged KV.  Unlike the
 // decode step this is a dense contraction, so it runs on tcgen05.mma:
 //
-//  * One CTA per work item (trajectory b, KV head g, 256 query rows).  A row
-//    is a (query token, query head of group g) pair, token-major, so the G
-//    heads sharing a KV head share every K/V tile (GQA).  The 256 rows form
-//    two 128-row tiles, A and B, that share each K/V tile: every K/V byte
-//    brought into shared memory feeds twice the MMA work.
-//  * Warp 0 (TMA producer) loads the two Q tiles once (3-D tensor map, two
-//    64-column panels each, 128-byte swizzle) and streams K and V tiles of 128
-//    keys (8 pages, two 2 KB boxes per page and operand, issued from 32 lanes
-//    at once) into a 3-stage K ring and a 2-stage V ring; K is released as
-//    soon as both S MMAs have read it, so it is loaded a tile ahead of V.
+//  * A work item is (trajectory b, KV head g, query block of two 128-row
+//    tiles A and B).  A row is a (query token, query head of group g) pair,
+//    token-major, so the G heads sharing a KV head share every K/V tile (GQA),
+//    and tiles A and B share each K/V tile: every K/V byte brought into shared
+//    memory feeds twice the MMA work.
+//  * Persistent CTAs, one per SM, pull work units in order from a counter:
+//    first whole items (so the query blocks of a (trajectory, KV head) run
+//    side by side and share its K/V through L2), then the items of the last
+//    partial wave cut into pieces of their key tiles, about one per CTA, so
+//    that the CTAs that finish first take the remaining work and no SM idles
+//    through a last partial wave.  Each piece stores its rows' O / l and
+//    log2-lse; the CTA that completes an item last merges its pieces in piece
+//    order (deterministic).  Within a CTA the producer warp fetches the units
+//    and hands them to the other warps through a small ring; every ring and
+//    barrier phase counts the CTA's key tiles or units, so the pipelines run
+//    on from one unit to the next.
+//  * Warp 10 loads each segment's two Q tiles (3-D tensor map, two 64-column
+//    panels each, 128-byte swizzle) once the previous segment's S MMAs are
+//    done.  Warp 0 streams K and V tiles of 128 keys (8 pages, two 2 KB boxes
+//    per page and operand, issued from 32 lanes at once) into a 3-stage K ring
+//    and a 2-stage V ring; K is released as soon as both S MMAs have read it,
+//    so it is loaded a tile ahead of V.
 //  * Warp 1 (MMA issuer, one lane) keeps S_A, S_B, O_A, O_B in TMEM (4 x 128
 //    fp32 columns).  Per key tile j it issues S_X = Q_X K_j^T and, once the
 //    softmax has turned S_X into P_X, O_X += P_X V_j with P_X read straight
@@ -27,8 +39,8 @@
 //    only on tiles that cross the diagonal, running max with lazy O rescaling
 //    (only when the max grows by more than 2^8; the decision is warp-uniform
 //    since tcgen05.ld/st are warp-collective), P = 2^(s - m) packed to bf16
-//    and stored with tcgen05.st over the S columns already consumed.  Finally
-//    O / l and lse.
+//    and stored with tcgen05.st over the S columns already consumed.  At the
+//    end of a segment: O / l and lse, or the piece's partial row.
 //  * All waits are bounded; on timeout the kernel records CADKV_ERR_TIMEOUT,
 //    waits for its own copies and MMAs, frees TMEM and returns.
 #include <cfloat>
@@ -47,26 +59,52 @@ constexpr unsigned kFull = 0xffffffffu;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kRows = 128;               // query rows per tile = MMA M
 constexpr int kTiles = 2;                // query tiles per CTA (A and B)
-constexpr int kItemRows = kRows * kTiles;
 constexpr int kKeys = 128;               // keys per tile = MMA N of QK^T, K of PV
 constexpr int kD = 128;                  // head_dim
 constexpr int kPanel = 16384;            // 128 rows x 128 B (one 64-column panel)
 constexpr int kTileBytes = 2 * kPanel;   // 128 rows x 128 columns bf16
 constexpr int kPageBlock = kPageSize * kD * 2;  // one (page, head) block: 4 KB
 constexpr int kSoftmaxThreads = 128 * kTiles;   // one warpgroup per query tile
-constexpr int kPrefillThreads = 64 + kSoftmaxThreads;  // producer, MMA, softmax
+// Warpgroup 0: K/V producer (warp 0), MMA issuer (1), Q loader (2), spare (3);
+// warpgroups 1 and 2: softmax of query tiles A and B.
+constexpr int kQLoaderWarp = 2;
+constexpr int kFirstSoftmaxWarp = 4;
+constexpr int kPrefillThreads = 128 + kSoftmaxThreads;
+// registers per thread after the split (launch: 168 for 384 threads; the
+// sum 128 * 152 + 256 * 176 equals the 384 * 168 the CTA holds)
+constexpr int kControlRegs = 152;
+constexpr int kSoftmaxRegs = 176;
+static_assert(128 * kControlRegs + kSoftmaxThreads * kSoftmaxRegs <= kPrefillThreads * 168,
+              "register split exceeds the launch allocation");
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 constexpr int kKStages = 3;              // K is freed early (after S), so it runs further ahead
 constexpr int kVStages = 2;
+constexpr int kUnitRing = 4;                 // work units handed from the producer to the other warps
+constexpr int kUnitReaders = 2 + kSoftmaxThreads / 32;  // Q loader, MMA issuer, softmax warps
+constexpr int kMaxPieces = 16;
+
+// A run of key tiles [kt0, kt1) of one work item.
+struct Segment {
+    long long q0;            // first query row of trajectory b
+    int b, g, qt;            // trajectory, KV head, query block
+    int kt0, kt1, num_kt;    // this run, and the item's key tile count
+    int i0, valid_tokens, chunk_start, pos_max, last_page;
+    int split;               // index of the split item, or -1 for a whole item
+    int piece;               // piece of the split item
+};
 
 struct PrefillSmem {
     uint8_t q[kTiles][kTileBytes];
     uint8_t k[kKStages][kTileBytes];
     uint8_t v[kVStages][kTileBytes];
-    uint64_t q_full, s_full[kTiles], p_full[kTiles], o_done[kTiles], k_full[kKStages],
-        k_empty[kKStages], v_full[kVStages], v_empty[kVStages], mma_done;
+    uint64_t q_full, q_empty, s_full[kTiles], p_full[kTiles], o_done[kTiles], k_full[kKStages],
+        k_empty[kKStages], v_full[kVStages], v_empty[kVStages], mma_done, part_written,
+        merge_decided, unit_full[kUnitRing], unit_empty[kUnitRing];
     uint32_t tmem_base;
     int abort;
+    int merge_last;
+    Segment unit_seg[kUnitRing];  // work units decoded by the producer warp
+    int unit_end[kUnitRing];      // 1: no more work
 };
 
 __device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo)
@@ -153,34 +191,105 @@ __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
+// ------------------------------------------------------------------ work split
+
+// Key tiles of query block qt of a trajectory whose chunk of C tokens ends at
+// position n - 1; block qt holds chunk tokens [qt * tpi, min((qt + 1) * tpi, C)).
+__device__ __forceinline__ int block_key_tiles(int n, int C, int tpi, int qt)
+{
+    const int end = n - C + min((qt + 1) * tpi, C);  // one past the block's last position
+    return (end + kKeys - 1) / kKeys;
+}
+
+
+// Work item i: trajectory b, KV head g, query block qt (items are ordered by
+// trajectory, then KV head, then query block), all its key tiles.
+__device__ Segment item_segment(const PrefillParams &p, long long i, int tokens_per_tile)
+{
+    Segment s;
+    int lo_b = 0, hi_b = p.batch - 1;
+    while (lo_b < hi_b) {  // largest b with item_prefix[b] <= i: never an empty trajectory
+        const int mid = (lo_b + hi_b + 1) >> 1;
+        if (p.item_prefix[mid] <= i)
+            lo_b = mid;
+        else
+            hi_b = mid - 1;
+    }
+    s.b = lo_b;
+    s.q0 = p.q_offsets[s.b];
+    const int C = (int)(p.q_offsets[s.b + 1] - s.q0);
+    const int n = p.context_lens[s.b];
+    const int tpi = kTiles * tokens_per_tile;
+    const int qblocks = (C + tpi - 1) / tpi;
+    const int local = (int)(i - p.item_prefix[s.b]);
+    s.g = local / qblocks;
+    s.qt = local - s.g * qblocks;
+    s.num_kt = block_key_tiles(n, C, tpi, s.qt);
+    s.kt0 = 0;
+    s.kt1 = s.num_kt;
+    s.i0 = s.qt * tpi;
+    s.valid_tokens = min(tpi, C - s.i0);
+    s.chunk_start = n - C;
+    s.pos_max = s.chunk_start + s.i0 + s.valid_tokens - 1;
+    s.last_page = s.pos_max / kPageSize;
+    s.split = -1;
+    s.piece = 0;
+    return s;
+}
+
+// Piece k of an item of nk key tiles split `pieces` ways: tiles
+// [k nk / pieces, (k + 1) nk / pieces); empty when nk < pieces for some k.
+__device__ __forceinline__ int piece_begin(int k, int nk, int pieces)
+{
+    return (int)((long long)k * nk / pieces);
+}
+
+// Work unit u: items [0, dp_items) whole, then piece (u - dp_items) % pieces
+// of split item dp_items + (u - dp_items) / pieces.  False for an empty piece.
+__device__ bool unit_segment(const PrefillParams &p, long long dp_items, int pieces, long long u,
+                             int tokens_per_tile, Segment &s)
+{
+    if (u < dp_items) {
+        s = item_segment(p, u, tokens_per_tile);
+        return true;
+    }
+    const long long v = u - dp_items;
+    const int split = (int)(v / pieces), k = (int)(v - (long long)split * pieces);
+    s = item_segment(p, dp_items + split, tokens_per_tile);
+    s.kt0 = piece_begin(k, s.num_kt, pieces);
+    s.kt1 = piece_begin(k + 1, s.num_kt, pieces);
+    s.split = split;
+    s.piece = k;
+    return s.kt0 < s.kt1;
+}
+
+// The CTA's k-th segment as the producer warp decoded and published it
+// (bounded wait); false at the end of the work or when the wait gave up.  The
+// caller releases the ring slot once it has read it.
+__device__ __forceinline__ bool read_segment(PrefillSmem &sm, long long k, volatile int *abort_flag,
+                                             bool &ok, Segment &sg)
+{
+    const int slot = (int)(k % kUnitRing);
+    ok = mbar_wait(&sm.unit_full[slot], (uint32_t)(k / kUnitRing) & 1, abort_flag);
+    if (!ok || sm.unit_end[slot])
+        return false;
+    sg = sm.unit_seg[slot];
+    return true;
+}
+
 // ------------------------------------------------------------------ planner
 
-__global__ void __launch_bounds__(1024, 1) prefill_plan_kernel(const PrefillParams p)
+// In-place exclusive scan of a[0..n) by one 1024-thread block; a[n] = total.
+__device__ void block_exclusive_scan(long long *a, int n, long long *warp_sums, long long *carry)
 {
-    __shared__ long long warp_sums[32];
-    __shared__ long long carry_s;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    if (tid == 0) {
-        p.hdr->status = 0;
-        carry_s = 0;
-    }
+    if (tid == 0)
+        *carry = 0;
     __syncthreads();
-    for (int base = 0; base < p.batch; base += 1024) {
-        const int b = base + tid;
-        long long items = 0;
-        if (b < p.batch) {
-            const long long qa = p.q_offsets[b], qb = p.q_offsets[b + 1];
-            const long long c = qb - qa;
-            const int n = p.context_lens[b];
-            if (qa < 0 || qb > p.total_q || c < 0 || n < 0 || c > n ||
-                n > p.max_pages * kPageSize) {
-                record_status(&p.hdr->status, CADKV_ERR_SHAPE);
-            } else {
-                const long long tpi = prefill_tokens_per_item(p.group);
-                items = (long long)p.num_kv_heads * ((c + tpi - 1) / tpi);
-            }
-        }
-        long long v = items;
+    for (int base = 0; base < n; base += 1024) {
+        const int i = base + tid;
+        const long long x = i < n ? a[i] : 0;
+        long long v = x;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const long long u = __shfl_up_sync(kFull, v, o);
@@ -201,17 +310,81 @@ __global__ void __launch_bounds__(1024, 1) prefill_plan_kernel(const PrefillPara
             warp_sums[lane] = w;
         }
         __syncthreads();
-        const long long incl = carry_s + v + (warp > 0 ? warp_sums[warp - 1] : 0);
-        if (b < p.batch)
-            p.item_prefix[b] = incl - items;
+        const long long incl = *carry + v + (warp > 0 ? warp_sums[warp - 1] : 0);
+        if (i < n)
+            a[i] = incl - x;
         __syncthreads();
         if (tid == 1023)
-            carry_s = incl;
+            *carry = incl;
         __syncthreads();
     }
+    if (tid == 0)
+        a[n] = *carry;
+    __syncthreads();
+}
+
+__global__ void __launch_bounds__(1024, 1) prefill_plan_kernel(const PrefillParams p)
+{
+    __shared__ long long warp_sums[32];
+    __shared__ long long carry_s;
+    const int tid = threadIdx.x;
     if (tid == 0) {
-        p.item_prefix[p.batch] = carry_s;
-        p.hdr->total_work = carry_s;
+        p.hdr->status = 0;
+        p.hdr->slice_counter = 0;  // next work unit
+    }
+    for (int i = tid; i < p.num_ctas; i += 1024)
+        p.merge_counter[i] = 0;
+    const int tpi = kTiles * (kRows / p.group);
+    for (int b = tid; b < p.batch; b += 1024) {  // work items per trajectory
+        const long long qa = p.q_offsets[b], qb = p.q_offsets[b + 1];
+        const long long c = qb - qa;
+        const int n = p.context_lens[b];
+        long long qblocks = 0;
+        if (qa < 0 || qb > p.total_q || c < 0 || n < 0 || c > n || n > p.max_pages * kPageSize)
+            record_status(&p.hdr->status, CADKV_ERR_SHAPE);
+        else
+            qblocks = (c + tpi - 1) / tpi;
+        p.item_prefix[b] = (long long)p.num_kv_heads * qblocks;
+    }
+    __syncthreads();
+    block_exclusive_scan(p.item_prefix, p.batch, warp_sums, &carry_s);
+    // The items of the last partial wave (all of them when there are fewer
+    // items than CTAs) are cut into pieces; sum their key tiles in parallel.
+    __shared__ unsigned long long tail_tiles_s;
+    if (tid == 0)
+        tail_tiles_s = 0;
+    __syncthreads();
+    const long long items = p.item_prefix[p.batch];
+    const long long split = items >= p.num_ctas ? items % p.num_ctas : items;
+    for (long long i = items - split + tid; i < items; i += 1024) {
+        int lo_b = 0, hi_b = p.batch - 1;
+        while (lo_b < hi_b) {
+            const int mid = (lo_b + hi_b + 1) >> 1;
+            if (p.item_prefix[mid] <= i)
+                lo_b = mid;
+            else
+                hi_b = mid - 1;
+        }
+        const int C = (int)(p.q_offsets[lo_b + 1] - p.q_offsets[lo_b]);
+        const int qblocks = (C + tpi - 1) / tpi;
+        const int qt = (int)((i - p.item_prefix[lo_b]) % qblocks);
+        atomicAdd(&tail_tiles_s, (unsigned long long)block_key_tiles(p.context_lens[lo_b], C, tpi, qt));
+    }
+    __syncthreads();
+    if (tid == 0) {
+        // All pieces run in one round (split * pieces <= P): a second round, or
+        // merging many pieces, costs more than it balances.  At least 16 key
+        // tiles per piece.
+        long long pieces = 1;
+        if (split > 0) {
+            const long long per_item = (long long)tail_tiles_s / split;
+            pieces = min((long long)kMaxPieces, max(1ll, (long long)p.num_ctas / split));
+            pieces = min(pieces, max(1ll, per_item / 16));
+        }
+        p.hdr->total_items = items;
+        p.hdr->dp_items = items - split;
+        p.hdr->pieces = pieces;
+        p.hdr->total_work = items - split + split * pieces;  // work units
     }
 }
 
@@ -226,42 +399,20 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
     PrefillSmem &sm = *reinterpret_cast<PrefillSmem *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const long long total = p.hdr->total_work;
-    const long long item = blockIdx.x;
-    if (item >= total)
+    const long long units = p.hdr->total_work, dp_items = p.hdr->dp_items;
+    const int pieces = (int)p.hdr->pieces;
+    if (blockIdx.x >= units)
         return;  // uniform across the CTA, before any barrier or TMEM use
 
-    // ---- decode the work item: (trajectory b, KV head g, 256-row query block qt)
-    int lo = 0, hi = p.batch - 1;
-    while (lo < hi) {  // largest b with item_prefix[b] <= item
-        const int mid = (lo + hi + 1) >> 1;
-        if (p.item_prefix[mid] <= item)
-            lo = mid;
-        else
-            hi = mid - 1;
-    }
-    const int b = lo;
     const int G = p.group;
     // a tile holds floor(128 / G) whole tokens (all G heads of each); for G that
     // does not divide 128 the last 128 mod G rows are padding, never written out
     const int tokens_per_tile = kRows / G;
     const int rows_used = tokens_per_tile * G;
-    const long long q0 = p.q_offsets[b];
-    const int chunk = (int)(p.q_offsets[b + 1] - q0);
-    const int n = p.context_lens[b];
-    const int qblocks = (chunk + kTiles * tokens_per_tile - 1) / (kTiles * tokens_per_tile);
-    const int local = (int)(item - p.item_prefix[b]);
-    const int g = local / qblocks;
-    const int qt = qblocks - 1 - local % qblocks;  // heaviest blocks first
-    const int i0 = qt * kTiles * tokens_per_tile;  // first token of tile A
-    const int valid_tokens = min(kTiles * tokens_per_tile, chunk - i0);
-    const int chunk_start = n - chunk;
-    const int pos_max = chunk_start + i0 + valid_tokens - 1;
-    const int num_kt = (pos_max + 1 + kKeys - 1) / kKeys;
-    const int last_page = pos_max / kPageSize;  // inclusive
 
     if (tid == 0) {
         mbar_init(&sm.q_full, 1);
+        mbar_init(&sm.q_empty, 1);
         for (int t = 0; t < kTiles; ++t) {
             mbar_init(&sm.s_full[t], 1);
             mbar_init(&sm.p_full[t], 128);
@@ -276,7 +427,14 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             mbar_init(&sm.v_empty[s], 1);
         }
         mbar_init(&sm.mma_done, 1);
+        mbar_init(&sm.part_written, kSoftmaxThreads);
+        mbar_init(&sm.merge_decided, 1);
+        for (int i = 0; i < kUnitRing; ++i) {
+            mbar_init(&sm.unit_full[i], 1);
+            mbar_init(&sm.unit_empty[i], kUnitReaders);
+        }
         sm.abort = 0;
+        sm.merge_last = 0;
         fence_mbarrier_init();
     }
     if (rows_used < kRows) {
@@ -302,68 +460,91 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
     // columns: S_A [0,128), S_B [128,256), O_A [256,384), O_B [384,512); P_X is
     // written over the first 64 columns of S_X (two bf16 per column).
     volatile int *abort_flag = &sm.abort;
-
+    // Registers move from the control warpgroup to the softmax warpgroups,
+    // which hold a row's 128 scores plus the segment state; each warpgroup
+    // changes its allocation at the top of its own branch.
+    if (warp < kFirstSoftmaxWarp) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kControlRegs));
     if (warp == 0) {
-        // ============================ TMA producer ============================
+        // ============================ K/V producer ============================
         bool ok = true;
-        // every (trajectory, KV head)'s K/V is re-read by all its query-block CTAs
+        // every (trajectory, KV head)'s K/V is re-read by all its query blocks
         const uint64_t policy = l2_evict_last_policy();
         if (lane == 0) {
-            prefetch_tensor_map(&qmap);
             prefetch_tensor_map(&kmap);
             prefetch_tensor_map(&vmap);
-            mbar_arrive_expect_tx(&sm.q_full, kTiles * 2 * rows_used * 128);
-            for (int t = 0; t < kTiles; ++t) {
-                const int qy = (int)(q0 + i0 + t * tokens_per_tile);
-                for (int h = 0; h < 2; ++h)
-                    tma_load_3d(sm.q[t] + h * kPanel, &qmap, h * 64, g * G, qy, &sm.q_full);
-            }
         }
-        // Step J issues K_J (lanes 0-15) and V_{J-1} (lanes 16-31): K is freed
-        // right after the S MMAs while V waits for PV, so each stream is gated
-        // only by its own ring and K runs a tile ahead.  Box = one 64-column
-        // panel of one page: page = (lane / 2) % 8, panel = lane % 2.
+        // Step J of a segment issues its K_J (lanes 0-15) and V_{J-1} (lanes
+        // 16-31): K is freed right after the S MMAs while V waits for PV, so each
+        // stream is gated only by its own ring and K runs a tile ahead.  Box =
+        // one 64-column panel of one page: page = (lane / 2) % 8, panel = lane % 2.
         const int op = lane >> 4, pg = (lane >> 1) & 7, hh = lane & 1;
-        int issued_k = 0, issued_v = 0;
-        for (int J = 0; J <= num_kt && ok; ++J) {
-            const int jk = J, jv = J - 1;
-            const bool do_k = jk < num_kt, do_v = jv >= 0;
-            const int pages_k = do_k ? min(kKeys / kPageSize, last_page + 1 - jk * (kKeys / kPageSize)) : 0;
-            const int pages_v = do_v ? min(kKeys / kPageSize, last_page + 1 - jv * (kKeys / kPageSize)) : 0;
+        int nk = 0, nv = 0;  // K and V tiles this CTA has loaded
+        for (long long k = 0; ok; ++k) {
+            // fetch the CTA's next non-empty work unit, decode it once and hand
+            // the segment to the other warps
+            const int slot = (int)(k % kUnitRing);
             if (lane == 0) {
-                if (do_k) {
-                    const int sk = jk % kKStages;
-                    if (jk >= kKStages)
-                        ok = mbar_wait(&sm.k_empty[sk], ((jk / kKStages) + 1) & 1, abort_flag);
-                    if (ok)
-                        mbar_arrive_expect_tx(&sm.k_full[sk], (uint32_t)pages_k * kPageBlock);
+                if (k >= kUnitRing)
+                    ok = mbar_wait(&sm.unit_empty[slot], (uint32_t)((k / kUnitRing) + 1) & 1, abort_flag);
+                int end = 1;
+                while (ok) {
+                    const long long u = atomicAdd(&p.hdr->slice_counter, 1);
+                    if (u >= units)
+                        break;
+                    if (unit_segment(p, dp_items, pieces, u, tokens_per_tile, sm.unit_seg[slot])) {
+                        end = 0;
+                        break;
+                    }
                 }
-                if (do_v && ok) {
-                    const int sv = jv % kVStages;
-                    if (jv >= kVStages)
-                        ok = mbar_wait(&sm.v_empty[sv], ((jv / kVStages) + 1) & 1, abort_flag);
-                    if (ok)
-                        mbar_arrive_expect_tx(&sm.v_full[sv], (uint32_t)pages_v * kPageBlock);
-                }
+                sm.unit_end[slot] = end;
+                mbar_arrive(&sm.unit_full[slot]);
             }
+            __syncwarp();
             ok = __shfl_sync(kFull, ok ? 1 : 0, 0) != 0;
-            if (!ok)
+            if (!ok || sm.unit_end[slot])
                 break;
-            const int jt = op == 0 ? jk : jv;
-            const int pages = op == 0 ? pages_k : pages_v;
-            if ((op == 0 ? do_k : do_v) && pg < pages) {
-                int phys = p.block_table[(size_t)b * p.max_pages + jt * (kKeys / kPageSize) + pg];
-                if (phys < 0 || phys >= p.num_pages) {
-                    record_status(&p.hdr->status, CADKV_ERR_OOB);
-                    phys = 0;
+            const Segment sg = sm.unit_seg[slot];
+            const int nseg = sg.kt1 - sg.kt0;
+            for (int J = 0; J <= nseg && ok; ++J) {
+                const bool do_k = J < nseg, do_v = J > 0;
+                const int ktk = sg.kt0 + J, ktv = ktk - 1;
+                const int pages_k = do_k ? min(kKeys / kPageSize, sg.last_page + 1 - ktk * (kKeys / kPageSize)) : 0;
+                const int pages_v = do_v ? min(kKeys / kPageSize, sg.last_page + 1 - ktv * (kKeys / kPageSize)) : 0;
+                const int sk = nk % kKStages, sv = nv % kVStages;
+                if (lane == 0) {
+                    if (do_k) {
+                        if (nk >= kKStages)
+                            ok = mbar_wait(&sm.k_empty[sk], (uint32_t)((nk / kKStages) + 1) & 1, abort_flag);
+                        if (ok)
+                            mbar_arrive_expect_tx(&sm.k_full[sk], (uint32_t)pages_k * kPageBlock);
+                    }
+                    if (do_v && ok) {
+                        if (nv >= kVStages)
+                            ok = mbar_wait(&sm.v_empty[sv], (uint32_t)((nv / kVStages) + 1) & 1, abort_flag);
+                        if (ok)
+                            mbar_arrive_expect_tx(&sm.v_full[sv], (uint32_t)pages_v * kPageBlock);
+                    }
                 }
-                const int y = (phys * p.num_kv_heads + g) * kPageSize;
-                uint8_t *dst = (op == 0 ? sm.k[jt % kKStages] : sm.v[jt % kVStages]) + hh * kPanel + pg * 2048;
-                tma_load_2d(dst, op == 0 ? &kmap : &vmap, hh * 64, y,
-                            op == 0 ? &sm.k_full[jt % kKStages] : &sm.v_full[jt % kVStages], policy);
+                ok = __shfl_sync(kFull, ok ? 1 : 0, 0) != 0;
+                if (!ok)
+                    break;
+                const int kt = op == 0 ? ktk : ktv;
+                const int pages = op == 0 ? pages_k : pages_v;
+                if ((op == 0 ? do_k : do_v) && pg < pages) {
+                    int phys = p.block_table[(size_t)sg.b * p.max_pages + kt * (kKeys / kPageSize) + pg];
+                    if (phys < 0 || phys >= p.num_pages) {
+                        record_status(&p.hdr->status, CADKV_ERR_OOB);
+                        phys = 0;
+                    }
+                    const int y = (phys * p.num_kv_heads + sg.g) * kPageSize;
+                    uint8_t *dst = (op == 0 ? sm.k[sk] : sm.v[sv]) + hh * kPanel + pg * 2048;
+                    tma_load_2d(dst, op == 0 ? &kmap : &vmap, hh * 64, y,
+                                op == 0 ? &sm.k_full[sk] : &sm.v_full[sv], policy);
+                }
+                nk += do_k;
+                nv += do_v;
             }
-            issued_k += do_k;
-            issued_v += do_v;
         }
         if (lane == 0) {
             if (!ok) {
@@ -372,11 +553,44 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             }
             // every copy this warp started must land before the CTA exits
             volatile int never = 0;
-            mbar_wait(&sm.q_full, 0, &never);
-            for (int j = max(0, issued_k - kKStages); j < issued_k; ++j)
-                mbar_wait(&sm.k_full[j % kKStages], (j / kKStages) & 1, &never);
-            for (int j = max(0, issued_v - kVStages); j < issued_v; ++j)
-                mbar_wait(&sm.v_full[j % kVStages], (j / kVStages) & 1, &never);
+            for (int j = max(0, nk - kKStages); j < nk; ++j)
+                mbar_wait(&sm.k_full[j % kKStages], (uint32_t)(j / kKStages) & 1, &never);
+            for (int j = max(0, nv - kVStages); j < nv; ++j)
+                mbar_wait(&sm.v_full[j % kVStages], (uint32_t)(j / kVStages) & 1, &never);
+        }
+        __syncwarp();
+    } else if (warp == kQLoaderWarp) {
+        // ============================ Q loader ============================
+        if (lane == 0) {
+            prefetch_tensor_map(&qmap);
+            bool ok = true;
+            int seg = 0;
+            for (long long k = 0; ok; ++k) {
+                Segment sg;
+                const bool work = read_segment(sm, k, abort_flag, ok, sg);
+                mbar_arrive(&sm.unit_empty[k % kUnitRing]);
+                if (!work)
+                    break;
+                // the previous segment's S MMAs must be done with the Q tiles
+                if (seg > 0)
+                    ok = mbar_wait(&sm.q_empty, (uint32_t)(seg - 1) & 1, abort_flag);
+                if (!ok)
+                    break;
+                mbar_arrive_expect_tx(&sm.q_full, kTiles * 2 * rows_used * 128);
+                for (int t = 0; t < kTiles; ++t) {
+                    const int qy = (int)(sg.q0 + sg.i0 + t * tokens_per_tile);
+                    for (int h = 0; h < 2; ++h)
+                        tma_load_3d(sm.q[t] + h * kPanel, &qmap, h * 64, sg.g * G, qy, &sm.q_full);
+                }
+                ++seg;
+            }
+            if (!ok) {
+                *abort_flag = 1;
+                record_status(&p.hdr->status, CADKV_ERR_TIMEOUT);
+            }
+            volatile int never = 0;
+            if (seg > 0)  // the last Q copy this lane started lands before the CTA exits
+                mbar_wait(&sm.q_full, (uint32_t)(seg - 1) & 1, &never);
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -388,7 +602,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             // every instruction it spends between MMAs can leave the tensor pipe
             // idle.  All operand descriptors share one high word (stride, fixed
             // bits, swizzle); their low words are computed here once and the
-            // issue loop below, unrolled over the ring stages, only selects them.
+            // issue loop below, dispatched on the ring stages, only selects them.
             const uint32_t d_hi = (uint32_t)(desc_sw128(smem_addr(sm.q[0]), 16, 1024) >> 32);
             uint32_t q_lo[kTiles][kD / 16], k_lo[kKStages][kD / 16], v_lo[kVStages][kKeys / 16];
 #pragma unroll
@@ -406,7 +620,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
 #pragma unroll
                 for (int st = 0; st < kVStages; ++st)
                     v_lo[st][k] = (uint32_t)desc_sw128(smem_addr(sm.v[st] + k * 2048), kPanel, 1024);
-            auto desc = [&](uint32_t lo) { return ((uint64_t)d_hi << 32) | lo; };
+            auto desc = [&](uint32_t lo_word) { return ((uint64_t)d_hi << 32) | lo_word; };
             auto issue_s = [&](int t, auto stage) {  // S_t = Q_t K^T from K stage `stage`
                 constexpr int st = decltype(stage)::value;
 #pragma unroll
@@ -420,53 +634,90 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                 for (int k = 0; k < kKeys / 16; ++k)  // keys 16k .. 16k+15 = P columns 8k ..
                     umma_ts(tmem + 256 + t * kRows, tmem + t * kRows + 8 * k, desc(v_lo[st][k]), id_pv,
                             (!first || k > 0) ? 1u : 0u);
-                umma_commit(&sm.o_done[t]);
             };
             using S0 = std::integral_constant<int, 0>;
             using S1 = std::integral_constant<int, 1>;
             using S2 = std::integral_constant<int, 2>;
-            static_assert(kKStages == 3 && kVStages == 2, "the issue loop is unrolled over 6 tiles");
-            bool ok = mbar_wait(&sm.q_full, 0, abort_flag) && mbar_wait(&sm.k_full[0], 0, abort_flag);
-            if (ok) {
-                tc_fence_after();
-                issue_s(0, S0{});
-                issue_s(1, S0{});
-                umma_commit(&sm.k_empty[0]);
-            }
-            // one key tile: V_j in V stage sv, K_{j+1} in K stage sk1
-            auto step = [&](int j, auto sv_c, auto sk1_c) {
+            static_assert(kKStages == 3 && kVStages == 2, "the issue loop dispatches on 6 ring phases");
+            bool ok = true;
+            // one key tile, the CTA's n-th, j-th of a segment of nseg tiles: V in V
+            // stage sv, the next tile's K in K stage sk1; ph_p = n & 1,
+            // ph_v = (n / 2) & 1 and ph_k1 = ((n + 1) / 3) & 1 are the phases
+            auto step = [&](uint32_t ph_p, uint32_t ph_v, uint32_t ph_k1, int j, int nseg, auto sv_c,
+                            auto sk1_c) {
                 constexpr int sv = decltype(sv_c)::value, sk1 = decltype(sk1_c)::value;
-                const bool more = j + 1 < num_kt;
-                // tile A: PV_A(j) once P_A(j) is in TMEM, then S_A(j+1) over it
-                ok = mbar_wait(&sm.p_full[0], j & 1, abort_flag) &&
-                     mbar_wait(&sm.v_full[sv], (j / kVStages) & 1, abort_flag) &&
-                     (!more || mbar_wait(&sm.k_full[sk1], ((j + 1) / kKStages) & 1, abort_flag));
+                const bool more = j + 1 < nseg;
+                // tile A: PV_A once P_A is in TMEM, then the next S_A over it
+                ok = mbar_wait(&sm.p_full[0], ph_p, abort_flag) &&
+                     mbar_wait(&sm.v_full[sv], ph_v, abort_flag) &&
+                     (!more || mbar_wait(&sm.k_full[sk1], ph_k1, abort_flag));
                 if (!ok)
                     return;
                 tc_fence_after();
                 issue_pv(0, j == 0, sv_c);
+                if (!more)
+                    umma_commit(&sm.o_done[0]);
                 if (more)
                     issue_s(0, sk1_c);
-                // tile B likewise; then V_j and K_{j+1} are no longer needed
-                ok = mbar_wait(&sm.p_full[1], j & 1, abort_flag);
+                // tile B likewise; then this V and the next K are no longer needed
+                ok = mbar_wait(&sm.p_full[1], ph_p, abort_flag);
                 if (!ok)
                     return;
                 tc_fence_after();
                 issue_pv(1, j == 0, sv_c);
+                if (!more)
+                    umma_commit(&sm.o_done[1]);
                 umma_commit(&sm.v_empty[sv]);
                 if (more) {
                     issue_s(1, sk1_c);
                     umma_commit(&sm.k_empty[sk1]);
+                    if (j + 2 == nseg)  // that was the segment's last S: Q is free
+                        umma_commit(&sm.q_empty);
                 }
             };
-            for (int j0 = 0; j0 < num_kt && ok; j0 += 6) {
-                // (j mod 2, (j + 1) mod 3) for j = j0 .. j0 + 5, j0 a multiple of 6
-                step(j0, S0{}, S1{});
-                if (ok && j0 + 1 < num_kt) step(j0 + 1, S1{}, S2{});
-                if (ok && j0 + 2 < num_kt) step(j0 + 2, S0{}, S0{});
-                if (ok && j0 + 3 < num_kt) step(j0 + 3, S1{}, S1{});
-                if (ok && j0 + 4 < num_kt) step(j0 + 4, S0{}, S2{});
-                if (ok && j0 + 5 < num_kt) step(j0 + 5, S1{}, S0{});
+            long long n0 = 0;  // key tiles of this CTA before the current segment
+            int seg = 0;
+            for (long long k = 0; ok; ++k) {
+                Segment sg;
+                const bool work = read_segment(sm, k, abort_flag, ok, sg);
+                mbar_arrive(&sm.unit_empty[k % kUnitRing]);
+                if (!work)
+                    break;
+                const int nseg = sg.kt1 - sg.kt0;
+                const int sk = (int)(n0 % kKStages);
+                ok = mbar_wait(&sm.q_full, (uint32_t)seg & 1, abort_flag) &&
+                     mbar_wait(&sm.k_full[sk], (uint32_t)(n0 / kKStages) & 1, abort_flag);
+                if (!ok)
+                    break;
+                tc_fence_after();
+                switch (sk) {
+                case 0: issue_s(0, S0{}); issue_s(1, S0{}); umma_commit(&sm.k_empty[0]); break;
+                case 1: issue_s(0, S1{}); issue_s(1, S1{}); umma_commit(&sm.k_empty[1]); break;
+                default: issue_s(0, S2{}); issue_s(1, S2{}); umma_commit(&sm.k_empty[2]); break;
+                }
+                if (nseg == 1)
+                    umma_commit(&sm.q_empty);
+                // ring phases of tile n0, then advanced one tile at a time (no
+                // divisions on the issuing lane's path)
+                uint32_t r6 = (uint32_t)(n0 % 6), ph_p = (uint32_t)n0 & 1,
+                         ph_v = (uint32_t)(n0 / kVStages) & 1, ph_k1 = (uint32_t)((n0 + 1) / kKStages) & 1;
+                for (int j = 0; j < nseg && ok; ++j) {
+                    // (n mod 2, (n + 1) mod 3) picks the V stage and the next K stage
+                    switch (r6) {
+                    case 0: step(ph_p, ph_v, ph_k1, j, nseg, S0{}, S1{}); break;
+                    case 1: step(ph_p, ph_v, ph_k1, j, nseg, S1{}, S2{}); break;
+                    case 2: step(ph_p, ph_v, ph_k1, j, nseg, S0{}, S0{}); break;
+                    case 3: step(ph_p, ph_v, ph_k1, j, nseg, S1{}, S1{}); break;
+                    case 4: step(ph_p, ph_v, ph_k1, j, nseg, S0{}, S2{}); break;
+                    default: step(ph_p, ph_v, ph_k1, j, nseg, S1{}, S0{}); break;
+                    }
+                    r6 = r6 == 5 ? 0 : r6 + 1;  // now (n + 1) mod 6
+                    ph_p ^= 1;
+                    ph_v ^= (r6 & 1) ^ 1;       // n + 1 even: (n + 1) / 2 advanced
+                    ph_k1 ^= (r6 == 2 || r6 == 5) ? 1 : 0;  // (n + 2) mod 3 == 0
+                }
+                n0 += nseg;
+                ++seg;
             }
             if (!ok) {
                 *abort_flag = 1;
@@ -478,128 +729,247 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             mbar_wait(&sm.mma_done, 0, &never);
         }
         __syncwarp();
+    }
     } else {
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kSoftmaxRegs));
         // ============================ softmax warps ============================
-        const int t = (warp - 2) >> 2;            // query tile: 0 (A) or 1 (B)
+        const int t = (warp - kFirstSoftmaxWarp) >> 2;  // query tile: 0 (A) or 1 (B)
         const int row = 32 * (warp & 3) + lane;   // TMEM lane = row of the tile
+        const int prow = t * kRows + row;         // row of the 256-row partial
         const uint32_t lane_base = (uint32_t)(32 * (warp & 3)) << 16;
         const uint32_t s_col = tmem + lane_base + t * kRows;
         const uint32_t o_col = tmem + lane_base + 256 + t * kRows;
-        const int token = t * tokens_per_tile + row / G, head = row % G;
-        const bool row_valid = row < rows_used && token < valid_tokens;
-        const int pos_row = row_valid ? chunk_start + i0 + token : pos_max;
-        const int pos_min = chunk_start + i0 + t * tokens_per_tile;  // first row of the tile
+        const int head = row % G;
+        const int token = t * tokens_per_tile + row / G;  // within the query block
         const float scale = p.scale_log2;
-        float m = -INFINITY, l = 0.f;
         bool ok = true;
-        for (int j = 0; j < num_kt && ok; ++j) {
-            ok = __all_sync(kFull, mbar_wait(&sm.s_full[t], j & 1, abort_flag));
-            if (!ok)
+        long long n0 = 0;
+        int seg = 0, pieces_done = 0;
+        for (long long k = 0; ok; ++k) {
+            bool got;
+            Segment sg;
+            const bool work = __all_sync(kFull, read_segment(sm, k, abort_flag, got, sg));
+            ok = __all_sync(kFull, got);
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&sm.unit_empty[k % kUnitRing]);
+            if (!work)
                 break;
-            tc_fence_after();
-            const int key0 = j * kKeys;
-            const bool full_tile = key0 + kKeys - 1 <= pos_min;  // no key masked for any row
-            // the row's 128 scores in one burst of loads, one wait
-            uint32_t r[kKeys];
-            CADKV_TMEM_LD32(s_col + 0, r);
-            CADKV_TMEM_LD32(s_col + 32, (r + 32));
-            CADKV_TMEM_LD32(s_col + 64, (r + 64));
-            CADKV_TMEM_LD32(s_col + 96, (r + 96));
-            tmem_wait_ld();
-            if (!full_tile) {  // causal mask on tiles that cross the diagonal
+            const int nseg = sg.kt1 - sg.kt0;
+            const bool row_valid = row < rows_used && token < sg.valid_tokens;
+            const int pos_row = row_valid ? sg.chunk_start + sg.i0 + token : sg.pos_max;
+            const int pos_min = sg.chunk_start + sg.i0 + t * tokens_per_tile;  // first row of the tile
+            float m = -INFINITY, l = 0.f;
+            for (int j = 0; j < nseg && ok; ++j) {
+                const long long n = n0 + j;
+                ok = __all_sync(kFull, mbar_wait(&sm.s_full[t], (uint32_t)n & 1, abort_flag));
+                if (!ok)
+                    break;
+                tc_fence_after();
+                const int kt = sg.kt0 + j;
+                const int key0 = kt * kKeys;
+                const bool full_tile = key0 + kKeys - 1 <= pos_min;  // no key masked for any row
+                // the row's 128 scores in one burst of loads, one wait
+                uint32_t r[kKeys];
+                CADKV_TMEM_LD32(s_col + 0, r);
+                CADKV_TMEM_LD32(s_col + 32, (r + 32));
+                CADKV_TMEM_LD32(s_col + 64, (r + 64));
+                CADKV_TMEM_LD32(s_col + 96, (r + 96));
+                tmem_wait_ld();
+                if (!full_tile) {  // causal mask on tiles that cross the diagonal
+#pragma unroll
+                    for (int e = 0; e < kKeys; ++e)
+                        if (key0 + e > pos_row)
+                            r[e] = __float_as_uint(-INFINITY);
+                }
+                float mx = -INFINITY;
 #pragma unroll
                 for (int e = 0; e < kKeys; ++e)
-                    if (key0 + e > pos_row)
-                        r[e] = __float_as_uint(-INFINITY);
-            }
-            float mx = -INFINITY;
-#pragma unroll
-            for (int e = 0; e < kKeys; ++e)
-                mx = fmaxf(mx, __uint_as_float(r[e]));
-            const float m_new = fmaxf(m, mx * scale);
-            // Lazy rescaling: keep the stale max unless some lane's grew past the
-            // threshold; the decision is warp-uniform (tcgen05.ld/st are collective).
-            const bool rescale = __any_sync(kFull, m_new > m + kRescaleThreshold);
-            const float alpha = rescale ? exp2_approx(m - m_new) : 1.f;  // 0 on the first tile
-            if (rescale) {
-                l *= alpha;
-                m = m_new;
-            }
-            // P = 2^(s*scale - m) as bf16 pairs, over S columns already read
-            // (masked scores are -inf, so their P is exactly 0)
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t packed[16];
-#pragma unroll
-                for (int e = 0; e < 32; e += 2) {
-                    const float p0 = exp2_approx(__uint_as_float(r[32 * c + e]) * scale - m);
-                    const float p1 = exp2_approx(__uint_as_float(r[32 * c + e + 1]) * scale - m);
-                    l += p0 + p1;
-                    packed[e >> 1] = pack_bf16x2(p0, p1);
+                    mx = fmaxf(mx, __uint_as_float(r[e]));
+                const float m_new = fmaxf(m, mx * scale);
+                // Lazy rescaling: keep the stale max unless some lane's grew past the
+                // threshold; the decision is warp-uniform (tcgen05.ld/st are collective).
+                // A row whose keys so far are all masked (a piece that starts past
+                // it) keeps m = -inf, l = 0 and P = 0.
+                const bool rescale = __any_sync(kFull, m_new > m + kRescaleThreshold);
+                const float alpha = (rescale && m_new > -INFINITY) ? exp2_approx(m - m_new) : 1.f;
+                if (rescale) {
+                    l *= alpha;
+                    m = m_new;
                 }
-                CADKV_TMEM_ST16(s_col + c * 16, packed);
+                const float m_use = m > -INFINITY ? m : 0.f;
+                // P = 2^(s*scale - m) as bf16 pairs, over S columns already read
+                // (masked scores are -inf, so their P is exactly 0)
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t packed[16];
+#pragma unroll
+                    for (int e = 0; e < 32; e += 2) {
+                        const float p0 = exp2_approx(__uint_as_float(r[32 * c + e]) * scale - m_use);
+                        const float p1 = exp2_approx(__uint_as_float(r[32 * c + e + 1]) * scale - m_use);
+                        l += p0 + p1;
+                        packed[e >> 1] = pack_bf16x2(p0, p1);
+                    }
+                    CADKV_TMEM_ST16(s_col + c * 16, packed);
+                }
+                // O_t is stable here (this S_t was issued after the previous PV_t)
+                // and is not read again before the next PV_t, which waits for p_full.
+                if (rescale && j > 0) {
+                    for (int c = 0; c < 4; ++c) {
+                        uint32_t o[32];
+                        CADKV_TMEM_LD32(o_col + c * 32, o);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 32; ++e)
+                            o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+                        CADKV_TMEM_ST32(o_col + c * 32, o);
+                    }
+                }
+                tmem_wait_st();
+                if (kt == sg.num_kt - 1 && t == 0) {
+                    // Zero V rows past pos_max: those keys may hold NaN (slots past n_b,
+                    // or pages never loaded) and 0 * NaN would poison the PV sums.
+                    // PV_B of this tile is issued after PV_A, which waits for this.
+                    const int sv = (int)(n % kVStages);
+                    ok = __all_sync(kFull, mbar_wait(&sm.v_full[sv], (uint32_t)(n / kVStages) & 1, abort_flag));
+                    if (!ok)
+                        break;
+                    if (key0 + row > sg.pos_max) {
+                        for (int h = 0; h < 2; ++h) {
+                            uint4 *rz = reinterpret_cast<uint4 *>(sm.v[sv] + h * kPanel + row * 128);
+#pragma unroll
+                            for (int c16 = 0; c16 < 8; ++c16)
+                                rz[c16] = make_uint4(0, 0, 0, 0);
+                        }
+                    }
+                    fence_proxy_async_smem();
+                }
+                tc_fence_before();
+                mbar_arrive(&sm.p_full[t]);
             }
-            // O_t is stable here (S_t(j) was issued after PV_t(j-1)) and is not read
-            // again before PV_t(j), which waits for this tile's p_full.
-            if (rescale && j > 0) {
+            // ---- end of segment: O / l -> out, lse; or the piece's partial row
+            if (ok) {
+                ok = __all_sync(kFull, mbar_wait(&sm.o_done[t], (uint32_t)seg & 1, abort_flag));
+                tc_fence_after();
+            }
+            const bool whole = sg.kt0 == 0 && sg.kt1 == sg.num_kt;  // uniform across the CTA
+            const size_t out_row = (size_t)(sg.q0 + sg.i0 + token) * p.num_q_heads + sg.g * G + head;
+            if (ok && whole) {
+                const float inv = 1.f / l;
+                __nv_bfloat16 *orow = p.out + out_row * kD;
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t o[32];
+                    CADKV_TMEM_LD32(o_col + c * 32, o);
+                    tmem_wait_ld();
+                    if (row_valid) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
+#pragma unroll
+                        for (int q4 = 0; q4 < 4; ++q4) {
+                            uint4 v;
+                            v.x = pack_bf16x2(__uint_as_float(o[8 * q4 + 0]) * inv, __uint_as_float(o[8 * q4 + 1]) * inv);
+                            v.y = pack_bf16x2(__uint_as_float(o[8 * q4 + 2]) * inv, __uint_as_float(o[8 * q4 + 3]) * inv);
+                            v.z = pack_bf16x2(__uint_as_float(o[8 * q4 + 4]) * inv, __uint_as_float(o[8 * q4 + 5]) * inv);
+                            v.w = pack_bf16x2(__uint_as_float(o[8 * q4 + 6]) * inv, __uint_as_float(o[8 * q4 + 7]) * inv);
+                            dst[q4] = v;
+                        }
+                    }
+                }
+                if (row_valid && p.lse)
+                    p.lse[out_row] = (m + __log2f(l)) * kLn2;
+            } else if (ok) {
+                // A piece of a split item: its rows go to the piece's own slot.
+                const int slot = sg.split * pieces + sg.piece;
+                const float inv = l > 0.f ? 1.f / l : 0.f;
+                float4 *po = reinterpret_cast<float4 *>(p.partial_o + ((size_t)slot * kSoftmaxThreads + prow) * kD);
                 for (int c = 0; c < 4; ++c) {
                     uint32_t o[32];
                     CADKV_TMEM_LD32(o_col + c * 32, o);
                     tmem_wait_ld();
 #pragma unroll
-                    for (int e = 0; e < 32; ++e)
-                        o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-                    CADKV_TMEM_ST32(o_col + c * 32, o);
+                    for (int q4 = 0; q4 < 8; ++q4)
+                        po[c * 8 + q4] = make_float4(
+                            __uint_as_float(o[4 * q4 + 0]) * inv, __uint_as_float(o[4 * q4 + 1]) * inv,
+                            __uint_as_float(o[4 * q4 + 2]) * inv, __uint_as_float(o[4 * q4 + 3]) * inv);
                 }
-            }
-            tmem_wait_st();
-            if (j == num_kt - 1 && t == 0) {
-                // Zero V rows past pos_max: those keys may hold NaN (slots past n_b,
-                // or pages never loaded) and 0 * NaN would poison the PV sums.
-                ok = __all_sync(kFull, mbar_wait(&sm.v_full[j % kVStages], (j / kVStages) & 1, abort_flag));
-                if (!ok)
-                    break;
-                if (key0 + row > pos_max) {
-                    for (int h = 0; h < 2; ++h) {
-                        uint4 *rz = reinterpret_cast<uint4 *>(sm.v[j % kVStages] + h * kPanel + row * 128);
+                p.partial_lambda[(size_t)slot * kSoftmaxThreads + prow] = l > 0.f ? m + __log2f(l) : -INFINITY;
+                __threadfence();
+                // the first softmax thread counts the piece once all 256 rows are out
+                tc_fence_before();
+                mbar_arrive(&sm.part_written);
+                const int nonempty = min(sg.num_kt, pieces);  // pieces holding key tiles
+                if (tid == 32 * kFirstSoftmaxWarp) {
+                    ok = mbar_wait(&sm.part_written, (uint32_t)pieces_done & 1, abort_flag);
+                    if (ok) {
+                        __threadfence();
+                        const int prev = atomicAdd(&p.merge_counter[sg.split], 1);
+                        sm.merge_last = prev == nonempty - 1;  // every other piece is out
+                        __threadfence();
+                    }
+                    mbar_arrive(&sm.merge_decided);
+                }
+                ok = ok && __all_sync(kFull, mbar_wait(&sm.merge_decided, (uint32_t)pieces_done & 1, abort_flag));
+                ++pieces_done;
+                if (ok && *reinterpret_cast<volatile int *>(&sm.merge_last)) {
+                    // this CTA completes the item: merge the pieces in piece order
+                    __threadfence();
+                    float lam_max = -INFINITY;
+                    for (int k2 = 0; k2 < pieces; ++k2) {
+                        if (piece_begin(k2, sg.num_kt, pieces) == piece_begin(k2 + 1, sg.num_kt, pieces))
+                            continue;
+                        const int s2 = sg.split * pieces + k2;
+                        lam_max = fmaxf(lam_max, __ldcg(p.partial_lambda + (size_t)s2 * kSoftmaxThreads + prow));
+                    }
+                    float wsum = 0.f;
+                    for (int k2 = 0; k2 < pieces; ++k2) {
+                        if (piece_begin(k2, sg.num_kt, pieces) == piece_begin(k2 + 1, sg.num_kt, pieces))
+                            continue;
+                        const int s2 = sg.split * pieces + k2;
+                        const float lam = __ldcg(p.partial_lambda + (size_t)s2 * kSoftmaxThreads + prow);
+                        wsum += lam > -INFINITY ? exp2_approx(lam - lam_max) : 0.f;
+                    }
+                    const float inv_w = 1.f / wsum;
+                    for (int c = 0; c < 4; ++c) {  // 32 columns at a time
+                        float acc[32];
 #pragma unroll
-                        for (int c16 = 0; c16 < 8; ++c16)
-                            rz[c16] = make_uint4(0, 0, 0, 0);
+                        for (int d = 0; d < 32; ++d)
+                            acc[d] = 0.f;
+                        for (int k2 = 0; k2 < pieces; ++k2) {
+                            if (piece_begin(k2, sg.num_kt, pieces) == piece_begin(k2 + 1, sg.num_kt, pieces))
+                                continue;
+                            const size_t r2 = (size_t)(sg.split * pieces + k2) * kSoftmaxThreads + prow;
+                            const float lam = __ldcg(p.partial_lambda + r2);
+                            const float w = lam > -INFINITY ? exp2_approx(lam - lam_max) : 0.f;
+                            const float4 *src = reinterpret_cast<const float4 *>(p.partial_o + r2 * kD + c * 32);
+#pragma unroll
+                            for (int q4 = 0; q4 < 8; ++q4) {
+                                const float4 v = __ldcg(src + q4);
+                                acc[4 * q4 + 0] += w * v.x;
+                                acc[4 * q4 + 1] += w * v.y;
+                                acc[4 * q4 + 2] += w * v.z;
+                                acc[4 * q4 + 3] += w * v.w;
+                            }
+                        }
+                        if (row_valid) {
+                            uint4 *dst = reinterpret_cast<uint4 *>(p.out + out_row * kD + c * 32);
+#pragma unroll
+                            for (int q8 = 0; q8 < 4; ++q8) {
+                                uint4 v;
+                                v.x = pack_bf16x2(acc[8 * q8 + 0] * inv_w, acc[8 * q8 + 1] * inv_w);
+                                v.y = pack_bf16x2(acc[8 * q8 + 2] * inv_w, acc[8 * q8 + 3] * inv_w);
+                                v.z = pack_bf16x2(acc[8 * q8 + 4] * inv_w, acc[8 * q8 + 5] * inv_w);
+                                v.w = pack_bf16x2(acc[8 * q8 + 6] * inv_w, acc[8 * q8 + 7] * inv_w);
+                                dst[q8] = v;
+                            }
+                        }
+                    }
+                    if (row_valid) {
+                        if (p.lse)
+                            p.lse[out_row] = (lam_max + __log2f(wsum)) * kLn2;
                     }
                 }
-                fence_proxy_async_smem();
             }
-            tc_fence_before();
-            mbar_arrive(&sm.p_full[t]);
-        }
-        // ---- epilogue: O / l -> out, lse
-        if (ok) {
-            ok = __all_sync(kFull, mbar_wait(&sm.o_done[t], (num_kt - 1) & 1, abort_flag));
-            tc_fence_after();
-        }
-        if (ok) {
-            const float inv = 1.f / l;
-            __nv_bfloat16 *orow = p.out + ((size_t)(q0 + i0 + token) * p.num_q_heads + g * G + head) * kD;
-            for (int c = 0; c < 4; ++c) {
-                uint32_t o[32];
-                CADKV_TMEM_LD32(o_col + c * 32, o);
-                tmem_wait_ld();
-                if (row_valid) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
-#pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) {
-                        uint4 v;
-                        v.x = pack_bf16x2(__uint_as_float(o[8 * q4 + 0]) * inv, __uint_as_float(o[8 * q4 + 1]) * inv);
-                        v.y = pack_bf16x2(__uint_as_float(o[8 * q4 + 2]) * inv, __uint_as_float(o[8 * q4 + 3]) * inv);
-                        v.z = pack_bf16x2(__uint_as_float(o[8 * q4 + 4]) * inv, __uint_as_float(o[8 * q4 + 5]) * inv);
-                        v.w = pack_bf16x2(__uint_as_float(o[8 * q4 + 6]) * inv, __uint_as_float(o[8 * q4 + 7]) * inv);
-                        dst[q4] = v;
-                    }
-                }
-            }
-            if (row_valid && p.lse)
-                p.lse[(size_t)(q0 + i0 + token) * p.num_q_heads + g * G + head] =
-                    (m + __log2f(l)) * kLn2;
+            n0 += nseg;
+            ++seg;
         }
         if (!ok && lane == 0) {
             *abort_flag = 1;
@@ -619,10 +989,8 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
 
 size_t prefill_smem_bytes() { return sizeof(PrefillSmem) + 1024; }
 
-__host__ __device__ long long prefill_tokens_per_item(int group) { return (long long)kTiles * (kRows / group); }
-
 cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, const CUtensorMap &kmap,
-                           const CUtensorMap &vmap, int grid, cudaStream_t stream)
+                           const CUtensorMap &vmap, cudaStream_t stream)
 {
     static bool configured = false;
     const size_t smem = prefill_smem_bytes();
@@ -635,9 +1003,9 @@ cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, cons
     }
     prefill_plan_kernel<<<1, 1024, 0, stream>>>(p);
     cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess || grid == 0)
+    if (e != cudaSuccess)
         return e;
-    prefill_attention_kernel<<<grid, kPrefillThreads, smem, stream>>>(p, qmap, kmap, vmap);
+    prefill_attention_kernel<<<p.num_ctas, kPrefillThreads, smem, stream>>>(p, qmap, kmap, vmap);
     return cudaGetLastError();
 }
 
