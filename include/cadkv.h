@@ -214,7 +214,9 @@ int decode_attention_status(const void *workspace, cadkv_stream_t stream);
 /* state cannot be used and the destination recomputes the prefix)           */
 /* ------------------------------------------------------------------------ */
 
-/* Bytes of workspace prefill_attention needs for `batch` trajectories. */
+/* Bytes of workspace prefill_attention needs for `batch` trajectories on the
+ * current device (it holds, besides per-trajectory counts, partial rows for
+ * two pieces per SM: about 0.26 MB per SM). */
 size_t prefill_attention_workspace_size(int batch);
 
 /*
@@ -230,8 +232,12 @@ size_t prefill_attention_workspace_size(int batch);
  *   lse        fp32 [total_q][num_q_heads] or NULL
  * Query row i of trajectory b sits at position p = n_b - C_b + i and attends
  * to keys 0 .. p:  out = softmax_t<=p(q . K_t / sqrt(D)) V,  lse = ln sum exp.
- * Runs on the tcgen05 tensor cores (accumulators in TMEM), one CTA per
- * (trajectory, KV head, tile of 128 (query token, head) rows).
+ * Runs on the tcgen05 tensor cores (accumulators in TMEM) with one
+ * persistent CTA per SM pulling work items (trajectory, KV head, block of 2 x
+ * 128 (query token, head) rows); the items of the last partial wave are cut
+ * into pieces of their key tiles whose partial rows are merged, in a fixed
+ * order, by the CTA that completes the item.  The workspace must not be used
+ * by two calls in flight at once.
  * Supported: head_dim 128, page_size 16, G = Hq / Hkv in 1..8 (the Qwen3
  * models of Sec. 6 have G = 4, 5 and 8).
  * A trajectory with C_b > n_b or n_b out of range is skipped (its rows are
