@@ -327,6 +327,10 @@ __global__ void __launch_bounds__(1024, 1) prefill_plan_kernel(const PrefillPara
 {
     __shared__ long long warp_sums[32];
     __shared__ long long carry_s;
+    // Let the attention kernel launch now: it sets up its barriers and tensor
+    // memory, then waits (griddepcontrol.wait) for this grid before it reads
+    // anything written here.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int tid = threadIdx.x;
     if (tid == 0) {
         p.hdr->status = 0;
@@ -399,11 +403,6 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
     PrefillSmem &sm = *reinterpret_cast<PrefillSmem *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const long long units = p.hdr->total_work, dp_items = p.hdr->dp_items;
-    const int pieces = (int)p.hdr->pieces;
-    if (blockIdx.x >= units)
-        return;  // uniform across the CTA, before any barrier or TMEM use
-
     const int G = p.group;
     // a tile holds floor(128 / G) whole tokens (all G heads of each); for G that
     // does not divide 128 the last 128 mod G rows are padding, never written out
@@ -460,6 +459,12 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
     // columns: S_A [0,128), S_B [128,256), O_A [256,384), O_B [384,512); P_X is
     // written over the first 64 columns of S_X (two bf16 per column).
     volatile int *abort_flag = &sm.abort;
+    // Everything above overlaps the planner (programmatic dependent launch);
+    // from here on its writes are visible.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const long long units = p.hdr->total_work, dp_items = p.hdr->dp_items;
+    const int pieces = (int)p.hdr->pieces;
+    if (blockIdx.x < units) {  // uniform across the CTA
     // Registers move from the control warpgroup to the softmax warpgroups,
     // which hold a row's 128 scores plus the segment state; each warpgroup
     // changes its allocation at the top of its own branch.
@@ -595,7 +600,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
         __syncwarp();
     } else if (warp == 1) {
         // ============================ MMA issuer ============================
-        if (lane == 0) {
+        {
             const uint32_t id_qk = idesc_bf16(kRows, kKeys, 0, 0);
             const uint32_t id_pv = idesc_bf16(kRows, kD, 0, 1);
             // The issuing lane shares its SM sub-partition with softmax warps, so
@@ -620,6 +625,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
 #pragma unroll
                 for (int st = 0; st < kVStages; ++st)
                     v_lo[st][k] = (uint32_t)desc_sw128(smem_addr(sm.v[st] + k * 2048), kPanel, 1024);
+            if (lane == 0) {
             auto desc = [&](uint32_t lo_word) { return ((uint64_t)d_hi << 32) | lo_word; };
             auto issue_s = [&](int t, auto stage) {  // S_t = Q_t K^T from K stage `stage`
                 constexpr int st = decltype(stage)::value;
@@ -727,6 +733,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             umma_commit(&sm.mma_done);
             volatile int never = 0;
             mbar_wait(&sm.mma_done, 0, &never);
+            }
         }
         __syncwarp();
     }
@@ -977,6 +984,8 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
         }
     }
 
+    }
+
     tc_fence_before();
     __syncthreads();
     if (warp == 1) {
@@ -1005,8 +1014,18 @@ cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, cons
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess)
         return e;
-    prefill_attention_kernel<<<p.num_ctas, kPrefillThreads, smem, stream>>>(p, qmap, kmap, vmap);
-    return cudaGetLastError();
+    // Programmatic dependent launch: the attention kernel's prologue overlaps the planner.
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(p.num_ctas);
+    cfg.blockDim = dim3(kPrefillThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, prefill_attention_kernel, p, qmap, kmap, vmap);
 }
 
 }  // namespace cadkv
