@@ -297,31 +297,54 @@ def time_append_step(batch, tensors, steps, warmup, stream):
 
 def e2e_loop(batch, tensors, steps, warmup, stream):
     """decode_attention through the C ABI with host inputs and outputs: every
-    step copies q, block_table and context_lens from pinned host memory, runs
-    the step and reads out and lse back to pinned host memory."""
+    step uploads q, block_table and context_lens from pinned host memory, runs
+    the step and downloads out and lse to pinned host memory.  As in a serving
+    loop, transfers overlap compute: the device inputs are double-buffered,
+    step i + 1's upload runs on a copy stream while step i computes, and step
+    i's download follows it on the copy stream (events order the three)."""
     q, k, v, bt, cl, out, lse, ws = tensors
+    device = q.device
     hq = batch.q.cpu().pin_memory()
     hbt = torch.from_numpy(batch.block_table).pin_memory()
     hcl = torch.from_numpy(batch.context_lens).pin_memory()
     hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
     hlse = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
+    bufs = [(q, bt, cl, out, lse),
+            (torch.empty_like(q), torch.empty_like(bt), torch.empty_like(cl),
+             torch.empty_like(out), torch.empty_like(lse))]
+    copy = torch.cuda.Stream(device)
+    uploaded = [torch.cuda.Event() for _ in range(2)]
+    computed = [torch.cuda.Event() for _ in range(2)]
 
-    def step():
-        with torch.cuda.stream(stream):
-            q.copy_(hq, non_blocking=True)
-            bt.copy_(hbt, non_blocking=True)
-            cl.copy_(hcl, non_blocking=True)
-            cadkv.decode_attention(q, k, v, bt, cl, out=out, lse=lse, workspace=ws,
+    def upload(i):
+        dq, dbt, dcl = bufs[i % 2][:3]
+        with torch.cuda.stream(copy):
+            if i >= 2:  # buffer reuse: step i - 2 must be done with it
+                copy.wait_event(computed[i % 2])
+            dq.copy_(hq, non_blocking=True)
+            dbt.copy_(hbt, non_blocking=True)
+            dcl.copy_(hcl, non_blocking=True)
+            uploaded[i % 2].record(copy)
+
+    def run(n):
+        upload(0)
+        for i in range(n):
+            dq, dbt, dcl, dout, dlse = bufs[i % 2]
+            stream.wait_event(uploaded[i % 2])
+            cadkv.decode_attention(dq, k, v, dbt, dcl, out=dout, lse=dlse, workspace=ws,
                                    stream=stream)
-            hout.copy_(out, non_blocking=True)
-            hlse.copy_(lse, non_blocking=True)
-        stream.synchronize()
+            computed[i % 2].record(stream)
+            if i + 1 < n:
+                upload(i + 1)
+            with torch.cuda.stream(copy):
+                copy.wait_event(computed[i % 2])
+                hout.copy_(dout, non_blocking=True)
+                hlse.copy_(dlse, non_blocking=True)
+        torch.cuda.synchronize(device)
 
-    for _ in range(warmup):
-        step()
+    run(warmup)
     t0 = time.perf_counter()
-    for _ in range(steps):
-        step()
+    run(steps)
     secs = (time.perf_counter() - t0) / steps
     h2d = hq.numel() * 2 + hbt.numel() * 4 + hcl.numel() * 4
     d2h = hout.numel() * 2 + hlse.numel() * 4
