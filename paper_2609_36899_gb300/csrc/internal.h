@@ -101,7 +101,7 @@ struct PrefillParams {
     long long *item_prefix;      // [batch + 1] work items of trajectories before b
     int *merge_counter;          // [num_ctas] pieces done of split item i
     float *partial_lambda;       // [2 * num_ctas][256] log2-lse of a piece's rows
-    float *partial_o;            // [2 * num_ctas][256][128] O / l of a piece's rows
+    float *partial_o;            // [2 * num_ctas][128][256] O / l of a piece's rows, column-major
     long long total_q;           // rows of q / out; offsets beyond it are rejected
     int batch, num_q_heads, num_kv_heads, group, max_pages, num_pages, num_ctas;
     float scale_log2;

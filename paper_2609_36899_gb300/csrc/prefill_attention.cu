@@ -887,16 +887,16 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                 // A piece of a split item: its rows go to the piece's own slot.
                 const int slot = sg.split * pieces + sg.piece;
                 const float inv = l > 0.f ? 1.f / l : 0.f;
-                float4 *po = reinterpret_cast<float4 *>(p.partial_o + ((size_t)slot * kSoftmaxThreads + prow) * kD);
+                // column-major ([column][row]): a warp's stores and the merge's loads
+                // cover 32 consecutive rows of one column (coalesced)
+                float *po = p.partial_o + (size_t)slot * kD * kSoftmaxThreads + prow;
                 for (int c = 0; c < 4; ++c) {
                     uint32_t o[32];
                     CADKV_TMEM_LD32(o_col + c * 32, o);
                     tmem_wait_ld();
 #pragma unroll
-                    for (int q4 = 0; q4 < 8; ++q4)
-                        po[c * 8 + q4] = make_float4(
-                            __uint_as_float(o[4 * q4 + 0]) * inv, __uint_as_float(o[4 * q4 + 1]) * inv,
-                            __uint_as_float(o[4 * q4 + 2]) * inv, __uint_as_float(o[4 * q4 + 3]) * inv);
+                    for (int e = 0; e < 32; ++e)
+                        po[(size_t)(c * 32 + e) * kSoftmaxThreads] = __uint_as_float(o[e]) * inv;
                 }
                 p.partial_lambda[(size_t)slot * kSoftmaxThreads + prow] = l > 0.f ? m + __log2f(l) : -INFINITY;
                 __threadfence();
@@ -943,18 +943,18 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                         for (int k2 = 0; k2 < pieces; ++k2) {
                             if (piece_begin(k2, sg.num_kt, pieces) == piece_begin(k2 + 1, sg.num_kt, pieces))
                                 continue;
-                            const size_t r2 = (size_t)(sg.split * pieces + k2) * kSoftmaxThreads + prow;
-                            const float lam = __ldcg(p.partial_lambda + r2);
+                            const int s2 = sg.split * pieces + k2;
+                            const float lam = __ldcg(p.partial_lambda + (size_t)s2 * kSoftmaxThreads + prow);
                             const float w = lam > -INFINITY ? exp2_approx(lam - lam_max) : 0.f;
-                            const float4 *src = reinterpret_cast<const float4 *>(p.partial_o + r2 * kD + c * 32);
+                            const float *src =
+                                p.partial_o + ((size_t)s2 * kD + c * 32) * kSoftmaxThreads + prow;
+                            float v[32];
 #pragma unroll
-                            for (int q4 = 0; q4 < 8; ++q4) {
-                                const float4 v = __ldcg(src + q4);
-                                acc[4 * q4 + 0] += w * v.x;
-                                acc[4 * q4 + 1] += w * v.y;
-                                acc[4 * q4 + 2] += w * v.z;
-                                acc[4 * q4 + 3] += w * v.w;
-                            }
+                            for (int e = 0; e < 32; ++e)  // all 32 loads in flight at once
+                                v[e] = __ldcg(src + (size_t)e * kSoftmaxThreads);
+#pragma unroll
+                            for (int e = 0; e < 32; ++e)
+                                acc[e] += w * v[e];
                         }
                         if (row_valid) {
                             uint4 *dst = reinterpret_cast<uint4 *>(p.out + out_row * kD + c * 32);
