@@ -298,6 +298,20 @@ int kv_prefix_load(const cadkv_pool *pool, const int32_t *block_table, int max_p
 int kv_prefix_stage_status(const void *workspace, cadkv_stream_t stream);
 
 /*
+ * Self-test of the failure path (no counterpart in the paper).  Every device
+ * wait in this library is bounded; when one gives up, the kernel records
+ * CADKV_ERR_TIMEOUT in its workspace status word, waits (bounded) for its own
+ * copies, frees its tensor memory and returns, so the CUDA context stays
+ * usable.  This call runs exactly that path on purpose: one CTA holds tensor
+ * memory and waits, with the library's bounded wait, on a barrier phase that
+ * nothing ever completes; after limit_ns (1 ns .. 2 s) it records the timeout
+ * and returns.  Afterwards kv_prefix_stage_status(workspace, stream) reads
+ * CADKV_ERR_TIMEOUT.  workspace: device, at least 64 bytes, 256-byte aligned.
+ */
+int cadkv_wait_selftest(long long limit_ns, void *workspace, size_t workspace_bytes,
+                        cadkv_stream_t stream);
+
+/*
  * Measuring aid (no counterpart in the paper): read `bytes` (a multiple of 16)
  * of device memory `buf` with 16-byte streaming loads and XOR them into the
  * device word *sink (8-byte aligned; the caller zeroes it).  The only DRAM

@@ -70,6 +70,7 @@ _SIGNATURES = {
     "prefill_attention": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I,
                                _P, _SZ, _P]),
     "prefill_attention_status": (_I, [_P, _P]),
+    "cadkv_wait_selftest": (_I, [ctypes.c_longlong, _P, _SZ, _P]),
 }
 
 _lib = None
@@ -420,6 +421,15 @@ def cadkv_hbm_read_probe(buf, sink, stream=None):
     rc = library().cadkv_hbm_read_probe(_ptr(buf), buf.numel() * buf.element_size(),
                                         _ptr(sink), _stream(stream, buf.device))
     _check("cadkv_hbm_read_probe", rc)
+
+
+def cadkv_wait_selftest(limit_ns: int, workspace, stream=None):
+    """Run the library's timeout path on purpose (see include/cadkv.h); the status
+    word in ``workspace`` then reads CADKV_ERR_TIMEOUT."""
+    _need(workspace, "workspace", torch.uint8, 1, None)
+    rc = library().cadkv_wait_selftest(int(limit_ns), _ptr(workspace), workspace.numel(),
+                                       _stream(stream, workspace.device))
+    _check("cadkv_wait_selftest", rc)
 
 
 def kv_prefix_stage_status(workspace, stream=None) -> int:

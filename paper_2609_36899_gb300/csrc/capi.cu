@@ -803,6 +803,22 @@ int kv_prefix_stage_status(const void *workspace, cadkv_stream_t stream)
     return read_status(workspace, reinterpret_cast<cudaStream_t>(stream));
 }
 
+int cadkv_wait_selftest(long long limit_ns, void *workspace, size_t workspace_bytes,
+                        cadkv_stream_t stream)
+{
+    if (limit_ns <= 0 || limit_ns > 2000000000ll)
+        return CADKV_ERR_INVALID;
+    if (!workspace || !aligned(workspace, kWorkspaceAlign) ||
+        workspace_bytes < sizeof(WorkspaceHeader))
+        return CADKV_ERR_WORKSPACE;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    WorkspaceHeader *hdr = static_cast<WorkspaceHeader *>(workspace);
+    if (cudaMemsetAsync(hdr, 0, sizeof(WorkspaceHeader), s) != cudaSuccess)
+        return CADKV_ERR_CUDA;
+    return launch_wait_selftest(hdr, (unsigned long long)limit_ns, s) == cudaSuccess ? CADKV_OK
+                                                                                       : CADKV_ERR_CUDA;
+}
+
 int cadkv_hbm_read_probe(const void *buf, size_t bytes, unsigned long long *sink,
                          cadkv_stream_t stream)
 {

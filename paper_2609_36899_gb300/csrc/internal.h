@@ -136,6 +136,8 @@ StageWorkspaceLayout stage_workspace_layout(int batch);
 
 cudaError_t launch_stage(const StageParams &p, int num_sms, cudaStream_t stream);
 
+cudaError_t launch_wait_selftest(WorkspaceHeader *hdr, unsigned long long limit_ns,
+                                 cudaStream_t stream);
 cudaError_t launch_hbm_read(const void *src, size_t bytes, unsigned long long *sink,
                             int num_sms, cudaStream_t stream);
 

@@ -70,8 +70,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
 }
 
 // Wait for phase `parity` of `bar` to complete.  Gives up (returns false) when
-// *abort becomes non-zero or after kWaitLimitNs; never spins forever.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort)
+// *abort becomes non-zero or after limit_ns; never spins forever.
+__device__ __forceinline__ bool mbar_wait_for(uint64_t *bar, uint32_t parity, volatile int *abort,
+                                              unsigned long long limit_ns)
 {
     if (mbar_try_wait(bar, parity))
         return true;
@@ -81,9 +82,15 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
             return true;
         if (*abort)
             return false;
-        if (global_timer_ns() - t0 > kWaitLimitNs)
+        if (global_timer_ns() - t0 > limit_ns)
             return false;
     }
+}
+
+// mbar_wait_for with the library's limit, kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort)
+{
+    return mbar_wait_for(bar, parity, abort, kWaitLimitNs);
 }
 
 // ---------------------------------------------------------------- TMA

@@ -262,3 +262,21 @@ def test_hbm_read_probe_reads_every_word():
     expect = int(np.bitwise_xor.reduce(host.numpy().view(np.uint32)))
     assert int(sink.item()) & 0xFFFFFFFF == expect
     assert int(sink.item()) >> 32 == 0
+
+
+def test_bounded_wait_gives_up_and_context_stays_usable():
+    """The failure path, run on purpose: a kernel holding tensor memory waits with
+    the library's bounded wait on a barrier phase nothing completes.  It must give
+    up after the limit, report CADKV_ERR_TIMEOUT in the status word, free its
+    resources and leave the context usable for the next call."""
+    import time
+    ws = torch.zeros(4096, dtype=torch.uint8, device="cuda")
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    cadkv.cadkv_wait_selftest(50_000_000, ws)            # 50 ms
+    assert cadkv.kv_prefix_stage_status(ws) == STATUS["CADKV_ERR_TIMEOUT"]
+    assert time.perf_counter() - t0 >= 0.045
+    batch = make_batch([5, 100, 1000], 8, 2, 128, seed=77)  # the next call still works
+    out, lse = gpu_decode(batch)
+    ref, ref_lse = oracle_decode(batch)
+    assert_close(out, lse, ref, ref_lse, "decode after the self-test")
