@@ -807,17 +807,30 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                 const float m_use = m > -INFINITY ? m : 0.f;
                 // P = 2^(s*scale - m) as bf16 pairs, over S columns already read
                 // (masked scores are -inf, so their P is exactly 0)
+                {
+                    // paired fp32 arithmetic (fma / add .f32x2): half the instructions
+                    // for s * scale - m and for the row sum, which also frees issue
+                    // slots for the MMA lane on the same sub-partition
+                    const uint64_t sc2 = ((uint64_t)__float_as_uint(scale) << 32) | __float_as_uint(scale);
+                    const uint64_t nm2 = ((uint64_t)__float_as_uint(-m_use) << 32) | __float_as_uint(-m_use);
+                    uint64_t l2 = 0;
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    uint32_t packed[16];
+                    for (int c = 0; c < 4; ++c) {
+                        uint32_t packed[16];
 #pragma unroll
-                    for (int e = 0; e < 32; e += 2) {
-                        const float p0 = exp2_approx(__uint_as_float(r[32 * c + e]) * scale - m_use);
-                        const float p1 = exp2_approx(__uint_as_float(r[32 * c + e + 1]) * scale - m_use);
-                        l += p0 + p1;
-                        packed[e >> 1] = pack_bf16x2(p0, p1);
+                        for (int e = 0; e < 32; e += 2) {
+                            const uint64_t x = ((uint64_t)r[32 * c + e + 1] << 32) | r[32 * c + e];
+                            uint64_t y;
+                            asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(y) : "l"(x), "l"(sc2), "l"(nm2));
+                            const float p0 = exp2_approx(__uint_as_float((uint32_t)y));
+                            const float p1 = exp2_approx(__uint_as_float((uint32_t)(y >> 32)));
+                            const uint64_t pp = ((uint64_t)__float_as_uint(p1) << 32) | __float_as_uint(p0);
+                            asm("add.f32x2 %0, %1, %2;" : "=l"(l2) : "l"(l2), "l"(pp));
+                            packed[e >> 1] = pack_bf16x2(p0, p1);
+                        }
+                        CADKV_TMEM_ST16(s_col + c * 16, packed);
                     }
-                    CADKV_TMEM_ST16(s_col + c * 16, packed);
+                    l += __uint_as_float((uint32_t)l2) + __uint_as_float((uint32_t)(l2 >> 32));
                 }
                 // O_t is stable here (this S_t was issued after the previous PV_t)
                 // and is not read again before the next PV_t, which waits for p_full.
