@@ -789,28 +789,16 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                         if (key0 + e > pos_row)
                             r[e] = __float_as_uint(-INFINITY);
                 }
-                float mx = -INFINITY;
-#pragma unroll
-                for (int e = 0; e < kKeys; ++e)
-                    mx = fmaxf(mx, __uint_as_float(r[e]));
-                const float m_new = fmaxf(m, mx * scale);
-                // Lazy rescaling: keep the stale max unless some lane's grew past the
-                // threshold; the decision is warp-uniform (tcgen05.ld/st are collective).
-                // A row whose keys so far are all masked (a piece that starts past
-                // it) keeps m = -inf, l = 0 and P = 0.
-                const bool rescale = __any_sync(kFull, m_new > m + kRescaleThreshold);
-                const float alpha = (rescale && m_new > -INFINITY) ? exp2_approx(m - m_new) : 1.f;
-                if (rescale) {
-                    l *= alpha;
-                    m = m_new;
-                }
-                const float m_use = m > -INFINITY ? m : 0.f;
-                // P = 2^(s*scale - m) as bf16 pairs, over S columns already read
-                // (masked scores are -inf, so their P is exactly 0)
-                {
-                    // paired fp32 arithmetic (fma / add .f32x2): half the instructions
-                    // for s * scale - m and for the row sum, which also frees issue
-                    // slots for the MMA lane on the same sub-partition
+                // P = 2^(s*scale - m) against the running max m, without a max pass:
+                // while every P stays below 2^8 (the tile's row sum bounds them) m is
+                // kept; otherwise (and on a row's first tile) the max is taken, m
+                // moves to it and P is recomputed.  Masked scores are -inf: P = 0.
+                bool rescale = false;
+                float alpha = 1.f;
+                float lt = 0.f;
+                bool fresh = __any_sync(kFull, !(m > -INFINITY));
+                if (!fresh) {
+                    const float m_use = m;
                     const uint64_t sc2 = ((uint64_t)__float_as_uint(scale) << 32) | __float_as_uint(scale);
                     const uint64_t nm2 = ((uint64_t)__float_as_uint(-m_use) << 32) | __float_as_uint(-m_use);
                     uint64_t l2 = 0;
@@ -830,8 +818,43 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                         }
                         CADKV_TMEM_ST16(s_col + c * 16, packed);
                     }
-                    l += __uint_as_float((uint32_t)l2) + __uint_as_float((uint32_t)(l2 >> 32));
+                    lt = __uint_as_float((uint32_t)l2) + __uint_as_float((uint32_t)(l2 >> 32));
+                    fresh = __any_sync(kFull, !(lt <= 256.f));
                 }
+                if (fresh) {
+                    float mx = -INFINITY;
+#pragma unroll
+                    for (int e = 0; e < kKeys; ++e)
+                        mx = fmaxf(mx, __uint_as_float(r[e]));
+                    const float m_new = fmaxf(m, mx * scale);
+                    // a row whose keys so far are all masked keeps m = -inf, l = 0, P = 0
+                    rescale = __any_sync(kFull, m_new > m);
+                    alpha = (m_new > m && m_new > -INFINITY) ? exp2_approx(m - m_new) : 1.f;
+                    l *= alpha;
+                    m = fmaxf(m, m_new);
+                    const float m_use = m > -INFINITY ? m : 0.f;
+                    const uint64_t sc2 = ((uint64_t)__float_as_uint(scale) << 32) | __float_as_uint(scale);
+                    const uint64_t nm2 = ((uint64_t)__float_as_uint(-m_use) << 32) | __float_as_uint(-m_use);
+                    uint64_t l2 = 0;
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        uint32_t packed[16];
+#pragma unroll
+                        for (int e = 0; e < 32; e += 2) {
+                            const uint64_t x = ((uint64_t)r[32 * c + e + 1] << 32) | r[32 * c + e];
+                            uint64_t y;
+                            asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(y) : "l"(x), "l"(sc2), "l"(nm2));
+                            const float p0 = exp2_approx(__uint_as_float((uint32_t)y));
+                            const float p1 = exp2_approx(__uint_as_float((uint32_t)(y >> 32)));
+                            const uint64_t pp = ((uint64_t)__float_as_uint(p1) << 32) | __float_as_uint(p0);
+                            asm("add.f32x2 %0, %1, %2;" : "=l"(l2) : "l"(l2), "l"(pp));
+                            packed[e >> 1] = pack_bf16x2(p0, p1);
+                        }
+                        CADKV_TMEM_ST16(s_col + c * 16, packed);
+                    }
+                    lt = __uint_as_float((uint32_t)l2) + __uint_as_float((uint32_t)(l2 >> 32));
+                }
+                l += lt;
                 // O_t is stable here (this S_t was issued after the previous PV_t)
                 // and is not read again before the next PV_t, which waits for p_full.
                 if (rescale && j > 0) {

@@ -110,6 +110,31 @@ def test_prefill_full_size_sampled():
     torch.cuda.empty_cache()
 
 
+@pytest.mark.parametrize("direction", [1.0, -1.0])
+def test_prefill_running_max_moves(direction):
+    """Scores that rise (or fall) steadily along the context.  Rising: every key
+    tile lifts each row's max by ~16 log2 units, so P taken against the previous
+    max is far too large and must be recomputed against the new one.  Falling:
+    the first key tile holds the max throughout."""
+    lens, chunks = [1500, 700], [300, 129]
+    batch, offs, q = _case(lens, chunks, 2, 2, seed=460)
+    q.fill_(0.25)
+    kp = batch.k_pages.float()
+    for b, n in enumerate(lens):
+        npg = (n + 15) // 16
+        pages = torch.from_numpy(batch.block_table[b, :npg].astype(np.int64))
+        c = direction * torch.arange(n, dtype=torch.float32) / 16.0
+        for h in range(2):
+            blk = kp[pages, h].reshape(npg * 16, 128)    # a copy; slots past n stay NaN
+            blk[:n] = 0.5 * c[:, None] + 0.05 * blk[:n]  # aligned with q, plus noise
+            kp[pages, h] = blk.reshape(npg, 16, 128)
+    batch.k_pages = kp.to(torch.bfloat16)
+    out, lse, ws = _run(batch, offs, q)
+    assert cadkv.prefill_attention_status(ws) == 0
+    ref, ref_lse = _oracle(batch, offs, q)
+    assert_close(out, lse, ref, ref_lse, f"prefill, running max direction {direction}")
+
+
 def test_prefill_chunk_of_one_matches_decode():
     lens = [77, 1, 513]
     batch, offs, q = _case(lens, [1, 1, 1], 16, 2, seed=430)
