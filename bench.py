@@ -245,6 +245,85 @@ class OracleSample:
         return self._time(self.inputs)
 
 
+def oracle_staging_baseline(job, k_layers, v_layers, target_s=4.0):
+    """The oracle's prefix gather (C, OpenMP over the host cores) on a bounded
+    sample of the job's trajectories, one layer: GB/s read + write."""
+    import oracle
+    oracle.build()
+    orc = oracle.default()
+    threads = len(os.sched_getaffinity(0))
+    lens = job.context_lens
+    order = np.random.Generator(np.random.PCG64(STAGING.seed + 99)).permutation(len(lens))
+
+    def sample(chosen):
+        sel = lens[np.array(chosen)]
+        pages = -(-sel.astype(np.int64) // 16)
+        phys = np.concatenate([job.block_table[b, :pg] for b, pg in zip(chosen, pages)])
+        idx = torch.from_numpy(phys.astype(np.int64)).to(k_layers[0].device)
+        kp = bf16_bits(k_layers[0].index_select(0, idx))[None]
+        vp = bf16_bits(v_layers[0].index_select(0, idx))[None]
+        table = np.full((len(chosen), int(pages.max())), -1, dtype=np.int32)
+        pos = 0
+        for i, pg in enumerate(pages):
+            table[i, :pg] = np.arange(pos, pos + pg)
+            pos += pg
+        return kp, vp, table, sel
+
+    def timed(inp):
+        t0 = time.perf_counter()
+        orc.prefix_stage(inp[0], inp[1], inp[2], inp[3], 0, 1, num_threads=threads)
+        return time.perf_counter() - t0
+
+    pilot = sample([int(order[0])])
+    per_token = timed(pilot) / max(int(lens[order[0]]), 1)
+    chosen, tokens = [], 0
+    for b in order:
+        chosen.append(int(b))
+        tokens += int(lens[b])
+        if tokens * per_token >= target_s:
+            break
+    inp = sample(chosen)
+    secs = timed(inp)
+    nbytes = 2 * 2 * int(inp[3].sum()) * 8 * 128 * 2  # read + write, K and V, bytes
+    return {"value": round(nbytes / secs / 1e9, 3), "unit": "GB/s", "cores": threads,
+            "kind": "oracle", "seconds": round(secs, 2),
+            "sample": f"{len(chosen)} of {len(lens)} trajectories ({tokens} tokens), 1 layer, "
+                      f"C oracle gather, OpenMP {threads} threads"}
+
+
+def oracle_prefill_baseline(b, offs, q, w, target_s=4.0):
+    """The fp64 oracle (C, OpenMP over the host cores) on the last rows of
+    trajectory 0's chunk, every query head: TFLOP/s of algorithmic causal flops."""
+    import oracle
+    oracle.build()
+    orc = oracle.default()
+    threads = len(os.sched_getaffinity(0))
+    n = int(b.context_lens[0])
+    npg = -(-n // 16)
+    idx = torch.from_numpy(b.block_table[0, :npg].astype(np.int64)).to(b.k_pages.device)
+    kp = bf16_bits(b.k_pages.index_select(0, idx))
+    vp = bf16_bits(b.v_pages.index_select(0, idx))
+    table = np.arange(npg, dtype=np.int32)[None]
+    qb = bf16_bits(q[:w.chunk])
+
+    def run(rows):
+        sub = np.ascontiguousarray(qb[w.chunk - rows:])
+        t0 = time.perf_counter()
+        orc.prefill_attention(sub, np.array([0, rows], dtype=np.int64), kp, vp, table,
+                              np.array([n], dtype=np.int32), num_threads=threads)
+        return time.perf_counter() - t0
+
+    rows = max(1, min(w.chunk, int(target_s / max(run(4) / 4, 1e-9))))
+    secs = run(rows)
+    pos = np.arange(n - rows, n, dtype=np.float64)
+    flops = w.num_q_heads * float((4.0 * w.head_dim * (pos + 1)).sum())
+    return {"value": round(flops / secs / 1e12, 6), "unit": "TFLOP/s", "cores": threads,
+            "kind": "oracle", "seconds": round(secs, 2),
+            "sample": f"last {rows} of the {w.chunk} query tokens of trajectory 0 "
+                      f"(context {n}), all {w.num_q_heads} query heads, fp64 oracle, "
+                      f"OpenMP {threads} threads"}
+
+
 # ------------------------------------------------------------------ GPU legs
 
 def time_decode(tensors, steps, warmup, stream):
@@ -351,7 +430,7 @@ def e2e_loop(batch, tensors, steps, warmup, stream):
     return secs, h2d, d2h
 
 
-def bench_staging(device, reps, layers=2, batch=None):
+def bench_staging(device, reps, layers=2, batch=None, cpu_baseline=False):
     """Prefix staging of the staging workload's trajectories (all 64, or the
     first ``batch`` of the same draw) for ``layers`` layers (the full 48-layer
     job does not fit in HBM next to its destination; it runs as 48 / layers
@@ -419,6 +498,8 @@ def bench_staging(device, reps, layers=2, batch=None):
                         "unit": "GB/s", "frac": round(gbs / peak, 4),
                         "peak_kind": kind,
                         "traffic": profiled_traffic(STAGE_PROFILE_SUMMARY, STAGE_SOURCE)}}
+    if cpu_baseline:
+        res["cpu_baseline"] = oracle_staging_baseline(job, k_layers, v_layers)
     del dst, k_layers, v_layers, pool
     torch.cuda.empty_cache()
     return res
@@ -543,7 +624,7 @@ def bench_landscape(device, steps, warmup, batches=(8, 32, 128, 512),
     return cells
 
 
-def bench_prefill(device, steps, warmup):
+def bench_prefill(device, steps, warmup, cpu_baseline=False):
     """Chunked re-prefill: each of 8 trajectories recomputes attention for its
     last 512 tokens over a 16,384-token paged KV (32/8 heads, D=128)."""
     w = PREFILL
@@ -582,6 +663,8 @@ def bench_prefill(device, steps, warmup):
            "status": cadkv.prefill_attention_status(ws), "launches_per_call": 2,
            "roofline": {"bound": "tensor", "achieved": round(tflops, 1), "peak": peak,
                         "unit": "TFLOP/s", "frac": round(tflops / peak, 4), "peak_kind": kind}}
+    if cpu_baseline:
+        res["cpu_baseline"] = oracle_prefill_baseline(b, offs, q, w)
     del b, q, out
     torch.cuda.empty_cache()
     return res
@@ -657,13 +740,13 @@ def main():
     device = torch.device("cuda", torch.cuda.current_device())
     if args.workload == "staging":
         res = bench_staging(device, reps=args.steps, layers=args.staging_layers,
-                            batch=args.staging_batch)
+                            batch=args.staging_batch, cpu_baseline=not args.no_cpu_baseline)
         res["host"] = bench_host_staging(device, reps=args.steps)
         if rank == 0:
             print(json.dumps(res), flush=True)
         return
     if args.workload == "prefill":
-        res = bench_prefill(device, args.steps, args.warmup)
+        res = bench_prefill(device, args.steps, args.warmup, cpu_baseline=not args.no_cpu_baseline)
         if rank == 0:
             print(json.dumps(res), flush=True)
         return
@@ -762,8 +845,10 @@ def main():
     del batch, tensors
     torch.cuda.empty_cache()
     if rank == 0 and not args.no_extras:
-        line["staging"] = bench_staging(device, reps=10, layers=args.staging_layers)
+        line["staging"] = bench_staging(device, reps=10, layers=args.staging_layers,
+                                        cpu_baseline=not args.no_cpu_baseline)
         line["staging"]["host"] = bench_host_staging(device, reps=5)
+        line["prefill"] = bench_prefill(device, 10, 3, cpu_baseline=not args.no_cpu_baseline)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
