@@ -135,6 +135,18 @@ def test_prefill_running_max_moves(direction):
     assert_close(out, lse, ref, ref_lse, f"prefill, running max direction {direction}")
 
 
+def test_prefill_items_split_many_ways():
+    """Fewer work items than SMs, each with many key tiles: every item is cut into
+    the most pieces (16 here, 40,960 keys = 320 tiles per item), each piece stores
+    its partial rows and the last one to finish merges all of them."""
+    lens, chunks = [40960], [64]
+    batch, offs, q = _case(lens, chunks, 8, 1, seed=470)   # G = 8: 2 items of 32 tokens
+    out, lse, ws = _run(batch, offs, q)
+    assert cadkv.prefill_attention_status(ws) == 0
+    ref, ref_lse = _oracle(batch, offs, q)
+    assert_close(out, lse, ref, ref_lse, "prefill split 16 ways")
+
+
 def test_prefill_chunk_of_one_matches_decode():
     lens = [77, 1, 513]
     batch, offs, q = _case(lens, [1, 1, 1], 16, 2, seed=430)
