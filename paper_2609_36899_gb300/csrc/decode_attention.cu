@@ -155,8 +155,14 @@ __global__ void __launch_bounds__(1024, 1) plan_kernel(const PlanParams p)
         const long long W = total * p.num_kv_heads;
         const long long unit = p.slice_pages > 0 ? p.slice_pages : kMinSlicePages;
         long long T = (W + unit - 1) / unit;
-        if (T > p.slice_cap)
-            T = p.slice_cap;
+        // Dynamic slices (several per CTA) absorb per-SM speed differences, but
+        // each costs a start-up chain of dependent loads (slice, trajectory,
+        // table) and a pipeline fill; below ~4K page-heads per CTA that cost wins,
+        // so automatic slicing gives each CTA one equal slice there.
+        const long long ctas = p.slice_cap / kSlicesPerCta;
+        const long long cap = (p.slice_pages > 0 || W > kOneSliceMaxPerCta * ctas) ? p.slice_cap : ctas;
+        if (T > cap)
+            T = cap;
         if (T < 1)
             T = 1;
         p.hdr->total_work = W;

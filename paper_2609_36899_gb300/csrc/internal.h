@@ -18,6 +18,8 @@ constexpr int kAttnThreads = (kNumConsumerWarps + 1) * 32;
 constexpr int kSegRing = 8;        // segment descriptors in flight per CTA
 constexpr int kSlicesPerCta = 4;   // dynamic work slices per persistent CTA
 constexpr int kMinSlicePages = 16; // auto slicing never cuts finer than this
+constexpr long long kOneSliceMaxPerCta = 4096;  // page-heads per CTA up to which auto
+                                                // slicing gives each CTA a single slice
 constexpr size_t kWorkspaceAlign = 256;
 
 // Header at the start of a decode-attention or staging workspace.
