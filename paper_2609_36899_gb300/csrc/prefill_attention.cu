@@ -76,7 +76,7 @@ constexpr int kControlRegs = 152;
 constexpr int kSoftmaxRegs = 176;
 static_assert(128 * kControlRegs + kSoftmaxThreads * kSoftmaxRegs <= kPrefillThreads * 168,
               "register split exceeds the launch allocation");
-constexpr float kRescaleThreshold = 8.0f;  // log2 units
+constexpr float kMaxP = 256.f;  // P against a stale row max stays below 2^8
 constexpr int kKStages = 3;              // K is freed early (after S), so it runs further ahead
 constexpr int kVStages = 2;
 constexpr int kUnitRing = 4;                 // work units handed from the producer to the other warps
@@ -819,7 +819,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                         CADKV_TMEM_ST16(s_col + c * 16, packed);
                     }
                     lt = __uint_as_float((uint32_t)l2) + __uint_as_float((uint32_t)(l2 >> 32));
-                    fresh = __any_sync(kFull, !(lt <= 256.f));
+                    fresh = __any_sync(kFull, !(lt <= kMaxP));
                 }
                 if (fresh) {
                     float mx = -INFINITY;
