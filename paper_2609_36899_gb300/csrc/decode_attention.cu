@@ -8,8 +8,9 @@
 // Design (GB300-first):
 //  * Work = the flattened sequence of (trajectory b, KV head g, page j)
 //    "page-heads", ordered b-major.  A planner kernel computes the page prefix
-//    sum over trajectories; the sequence is cut into T equal slices, which a
-//    persistent grid (one CTA per SM) pulls with an atomic counter.  Equal
+//    sum over trajectories; the sequence is cut into T equal slices.  In a
+//    persistent grid (one CTA per SM) CTA i starts on slice i and pulls any
+//    further slice from an atomic counter.  Equal
 //    slices balance HBM bytes, not trajectories, so a few 128K-token tails and
 //    hundreds of 2K-token trajectories both keep every SM streaming.
 //  * Inside a CTA one producer warp issues TMA copies (cp.async.bulk.tensor,
@@ -82,6 +83,10 @@ __global__ void __launch_bounds__(1024, 1) plan_kernel(const PlanParams p)
     // waits (griddepcontrol.wait) for this whole grid to finish before it reads
     // anything the planner or the append CTAs write.
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    // This grid is itself launched programmatically, so it may start while the
+    // previous kernel on the stream (often the last decode step) is finishing:
+    // nothing is read or written here before that kernel's writes are visible.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     if (blockIdx.x > 0) {
         append_rows(p);
         return;
@@ -307,11 +312,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         uint32_t kp = 0;  // page-heads issued
         uint32_t sp = 0;  // segments issued
         bool ok = true;
-        while (ok) {
-            int slice = 0;
-            if (lane == 0)
-                slice = atomicAdd(&p.hdr->slice_counter, 1);
-            slice = __shfl_sync(kFull, slice, 0);
+        // Slice i < grid is CTA i's first; later slices come from the counter.
+        int slice = blockIdx.x;
+        for (bool initial = true; ok; initial = false) {
+            if (!initial) {
+                if (lane == 0)
+                    slice = (int)gridDim.x + atomicAdd(&p.hdr->slice_counter, 1);
+                slice = __shfl_sync(kFull, slice, 0);
+            }
             if (slice >= T)
                 break;
             const long long s0 = slice_begin(slice, W, T), s1 = slice_begin(slice + 1, W, T);
@@ -685,24 +693,27 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             const int slot0 = d.unit + d.first;
             for (int it = ct; it < G * (D / 8); it += kNumConsumerWarps * 32) {
                 const int h = it / (D / 8), d0 = (it % (D / 8)) * 8;
-                float M = -INFINITY;
-                for (int s2 = 0; s2 < d.count; ++s2)
-                    M = fmaxf(M, __ldcg(p.part_lse + (size_t)(slot0 + s2) * G + h));
-                float L = 0.f, acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                // One pass in slice order, rescaling the running sum as the max grows.
+                float M = -INFINITY, L = 0.f;
+                float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
                 for (int s2 = 0; s2 < d.count; ++s2) {
                     const size_t sl = (size_t)(slot0 + s2);
-                    const float w = exp2_approx(__ldcg(p.part_lse + sl * G + h) - M);
-                    L += w;
+                    const float lse_s = __ldcg(p.part_lse + sl * G + h);
                     const float4 *src = reinterpret_cast<const float4 *>(p.part_o + (sl * G + h) * D + d0);
                     const float4 u0 = __ldcg(src), u1 = __ldcg(src + 1);
-                    acc[0] += w * u0.x;
-                    acc[1] += w * u0.y;
-                    acc[2] += w * u0.z;
-                    acc[3] += w * u0.w;
-                    acc[4] += w * u1.x;
-                    acc[5] += w * u1.y;
-                    acc[6] += w * u1.z;
-                    acc[7] += w * u1.w;
+                    const float Mn = fmaxf(M, lse_s);
+                    const float a = exp2_approx(M - Mn), w = exp2_approx(lse_s - Mn);
+                    M = Mn;
+                    L = L * a + w;
+                    acc[0] = acc[0] * a + w * u0.x;
+                    acc[1] = acc[1] * a + w * u0.y;
+                    acc[2] = acc[2] * a + w * u0.z;
+                    acc[3] = acc[3] * a + w * u0.w;
+                    acc[4] = acc[4] * a + w * u1.x;
+                    acc[5] = acc[5] * a + w * u1.y;
+                    acc[6] = acc[6] * a + w * u1.z;
+                    acc[7] = acc[7] * a + w * u1.w;
                 }
                 const float inv = 1.f / L;
                 uint4 packed;
@@ -775,8 +786,19 @@ cudaError_t launch_plan(const PlanParams &p, cudaStream_t stream)
 {
     const int append_ctas =
         p.k_new ? (p.batch * p.num_kv_heads + kAppendRowsPerCta - 1) / kAppendRowsPerCta : 0;
-    plan_kernel<<<1 + append_ctas, 1024, 0, stream>>>(p);
-    return cudaGetLastError();
+    // Programmatic launch: the planner's start overlaps the previous kernel's
+    // tail; it waits for that kernel's writes before touching memory.
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(1 + append_ctas);
+    cfg.blockDim = dim3(1024);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, plan_kernel, p);
 }
 
 size_t attention_smem_bytes(int head_dim)
