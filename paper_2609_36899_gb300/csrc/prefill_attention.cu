@@ -71,9 +71,11 @@ constexpr int kQLoaderWarp = 2;
 constexpr int kFirstSoftmaxWarp = 4;
 constexpr int kPrefillThreads = 128 + kSoftmaxThreads;
 // registers per thread after the split (launch: 168 for 384 threads; the
-// sum 128 * 152 + 256 * 176 equals the 384 * 168 the CTA holds)
-constexpr int kControlRegs = 152;
-constexpr int kSoftmaxRegs = 176;
+// sum 128 * 120 + 256 * 192 equals the 384 * 168 the CTA holds).  The softmax
+// threads hold a row's 128 scores plus the segment state and spill below 192;
+// the control warps need far fewer.
+constexpr int kControlRegs = 120;
+constexpr int kSoftmaxRegs = 192;
 static_assert(128 * kControlRegs + kSoftmaxThreads * kSoftmaxRegs <= kPrefillThreads * 168,
               "register split exceeds the launch allocation");
 constexpr float kMaxP = 256.f;  // P against a stale row max stays below 2^8
@@ -607,52 +609,43 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             // every instruction it spends between MMAs can leave the tensor pipe
             // idle.  All operand descriptors share one high word (stride, fixed
             // bits, swizzle); their low words are computed here once and the
-            // issue loop below, dispatched on the ring stages, only selects them.
+            // issue loop below only offsets them: the ring stages are kTileBytes apart.
+            // (One step body for every stage keeps the issuing lane's code small.)
             const uint32_t d_hi = (uint32_t)(desc_sw128(smem_addr(sm.q[0]), 16, 1024) >> 32);
-            uint32_t q_lo[kTiles][kD / 16], k_lo[kKStages][kD / 16], v_lo[kVStages][kKeys / 16];
+            uint32_t q_lo[kTiles][kD / 16], k_lo[1][kD / 16], v_lo[1][kKeys / 16];
 #pragma unroll
             for (int k = 0; k < kD / 16; ++k) {
                 const int off = (k >> 2) * kPanel + (k & 3) * 32;
 #pragma unroll
                 for (int t = 0; t < kTiles; ++t)
                     q_lo[t][k] = (uint32_t)desc_sw128(smem_addr(sm.q[t] + off), 16, 1024);
-#pragma unroll
-                for (int st = 0; st < kKStages; ++st)
-                    k_lo[st][k] = (uint32_t)desc_sw128(smem_addr(sm.k[st] + off), 16, 1024);
+                k_lo[0][k] = (uint32_t)desc_sw128(smem_addr(sm.k[0] + off), 16, 1024);
             }
 #pragma unroll
             for (int k = 0; k < kKeys / 16; ++k)
-#pragma unroll
-                for (int st = 0; st < kVStages; ++st)
-                    v_lo[st][k] = (uint32_t)desc_sw128(smem_addr(sm.v[st] + k * 2048), kPanel, 1024);
+                v_lo[0][k] = (uint32_t)desc_sw128(smem_addr(sm.v[0] + k * 2048), kPanel, 1024);
             if (lane == 0) {
             auto desc = [&](uint32_t lo_word) { return ((uint64_t)d_hi << 32) | lo_word; };
-            auto issue_s = [&](int t, auto stage) {  // S_t = Q_t K^T from K stage `stage`
-                constexpr int st = decltype(stage)::value;
+            constexpr uint32_t kStage16 = kTileBytes >> 4;  // one ring stage in descriptor units
+            auto issue_s = [&](int t, uint32_t koff) {  // S_t = Q_t K^T from the K stage at koff
 #pragma unroll
                 for (int k = 0; k < kD / 16; ++k)
-                    umma_ss(tmem + t * kRows, desc(q_lo[t][k]), desc(k_lo[st][k]), id_qk, k > 0);
+                    umma_ss(tmem + t * kRows, desc(q_lo[t][k]), desc(k_lo[0][k] + koff), id_qk, k > 0);
                 umma_commit(&sm.s_full[t]);
             };
-            auto issue_pv = [&](int t, bool first, auto stage) {  // O_t += P_t V, P_t from TMEM
-                constexpr int st = decltype(stage)::value;
+            auto issue_pv = [&](int t, bool first, uint32_t voff) {  // O_t += P_t V, P_t from TMEM
 #pragma unroll
                 for (int k = 0; k < kKeys / 16; ++k)  // keys 16k .. 16k+15 = P columns 8k ..
-                    umma_ts(tmem + 256 + t * kRows, tmem + t * kRows + 8 * k, desc(v_lo[st][k]), id_pv,
+                    umma_ts(tmem + 256 + t * kRows, tmem + t * kRows + 8 * k, desc(v_lo[0][k] + voff), id_pv,
                             (!first || k > 0) ? 1u : 0u);
             };
-            using S0 = std::integral_constant<int, 0>;
-            using S1 = std::integral_constant<int, 1>;
-            using S2 = std::integral_constant<int, 2>;
-            static_assert(kKStages == 3 && kVStages == 2, "the issue loop dispatches on 6 ring phases");
             bool ok = true;
             // one key tile, the CTA's n-th, j-th of a segment of nseg tiles: V in V
-            // stage sv, the next tile's K in K stage sk1; ph_p = n & 1,
-            // ph_v = (n / 2) & 1 and ph_k1 = ((n + 1) / 3) & 1 are the phases
-            auto step = [&](uint32_t ph_p, uint32_t ph_v, uint32_t ph_k1, int j, int nseg, auto sv_c,
-                            auto sk1_c) {
-                constexpr int sv = decltype(sv_c)::value, sk1 = decltype(sk1_c)::value;
+            // stage sv = n % 2, the next tile's K in K stage sk1 = (n + 1) % 3;
+            // ph_p = n & 1, ph_v = (n / 2) & 1 and ph_k1 = ((n + 1) / 3) & 1 are the phases
+            auto step = [&](uint32_t ph_p, uint32_t ph_v, uint32_t ph_k1, int j, int nseg, int sv, int sk1) {
                 const bool more = j + 1 < nseg;
+                const uint32_t voff = (uint32_t)sv * kStage16, koff = (uint32_t)sk1 * kStage16;
                 // tile A: PV_A once P_A is in TMEM, then the next S_A over it
                 ok = mbar_wait(&sm.p_full[0], ph_p, abort_flag) &&
                      mbar_wait(&sm.v_full[sv], ph_v, abort_flag) &&
@@ -660,22 +653,22 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                 if (!ok)
                     return;
                 tc_fence_after();
-                issue_pv(0, j == 0, sv_c);
+                issue_pv(0, j == 0, voff);
                 if (!more)
                     umma_commit(&sm.o_done[0]);
                 if (more)
-                    issue_s(0, sk1_c);
+                    issue_s(0, koff);
                 // tile B likewise; then this V and the next K are no longer needed
                 ok = mbar_wait(&sm.p_full[1], ph_p, abort_flag);
                 if (!ok)
                     return;
                 tc_fence_after();
-                issue_pv(1, j == 0, sv_c);
+                issue_pv(1, j == 0, voff);
                 if (!more)
                     umma_commit(&sm.o_done[1]);
                 umma_commit(&sm.v_empty[sv]);
                 if (more) {
-                    issue_s(1, sk1_c);
+                    issue_s(1, koff);
                     umma_commit(&sm.k_empty[sk1]);
                     if (j + 2 == nseg)  // that was the segment's last S: Q is free
                         umma_commit(&sm.q_empty);
@@ -696,31 +689,23 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                 if (!ok)
                     break;
                 tc_fence_after();
-                switch (sk) {
-                case 0: issue_s(0, S0{}); issue_s(1, S0{}); umma_commit(&sm.k_empty[0]); break;
-                case 1: issue_s(0, S1{}); issue_s(1, S1{}); umma_commit(&sm.k_empty[1]); break;
-                default: issue_s(0, S2{}); issue_s(1, S2{}); umma_commit(&sm.k_empty[2]); break;
-                }
+                issue_s(0, (uint32_t)sk * kStage16);
+                issue_s(1, (uint32_t)sk * kStage16);
+                umma_commit(&sm.k_empty[sk]);
                 if (nseg == 1)
                     umma_commit(&sm.q_empty);
                 // ring phases of tile n0, then advanced one tile at a time (no
                 // divisions on the issuing lane's path)
-                uint32_t r6 = (uint32_t)(n0 % 6), ph_p = (uint32_t)n0 & 1,
-                         ph_v = (uint32_t)(n0 / kVStages) & 1, ph_k1 = (uint32_t)((n0 + 1) / kKStages) & 1;
+                uint32_t ph_p = (uint32_t)n0 & 1, ph_v = (uint32_t)(n0 / kVStages) & 1,
+                         ph_k1 = (uint32_t)((n0 + 1) / kKStages) & 1;
+                int sv = (int)(n0 & 1), sk1 = (int)((n0 + 1) % kKStages);
                 for (int j = 0; j < nseg && ok; ++j) {
-                    // (n mod 2, (n + 1) mod 3) picks the V stage and the next K stage
-                    switch (r6) {
-                    case 0: step(ph_p, ph_v, ph_k1, j, nseg, S0{}, S1{}); break;
-                    case 1: step(ph_p, ph_v, ph_k1, j, nseg, S1{}, S2{}); break;
-                    case 2: step(ph_p, ph_v, ph_k1, j, nseg, S0{}, S0{}); break;
-                    case 3: step(ph_p, ph_v, ph_k1, j, nseg, S1{}, S1{}); break;
-                    case 4: step(ph_p, ph_v, ph_k1, j, nseg, S0{}, S2{}); break;
-                    default: step(ph_p, ph_v, ph_k1, j, nseg, S1{}, S0{}); break;
-                    }
-                    r6 = r6 == 5 ? 0 : r6 + 1;  // now (n + 1) mod 6
+                    step(ph_p, ph_v, ph_k1, j, nseg, sv, sk1);
                     ph_p ^= 1;
-                    ph_v ^= (r6 & 1) ^ 1;       // n + 1 even: (n + 1) / 2 advanced
-                    ph_k1 ^= (r6 == 2 || r6 == 5) ? 1 : 0;  // (n + 2) mod 3 == 0
+                    ph_v ^= (uint32_t)sv;  // V stage 1 -> 0 wraps the ring
+                    sv ^= 1;
+                    sk1 = sk1 == kKStages - 1 ? 0 : sk1 + 1;
+                    ph_k1 ^= sk1 == 0 ? 1u : 0u;  // the next K stage wrapped
                 }
                 n0 += nseg;
                 ++seg;
