@@ -41,6 +41,7 @@ import paper_2609_36899_gb300 as cadkv  # noqa: E402
 from paper_2609_36899_gb300 import build as pkg_build  # noqa: E402
 from paper_2609_36899_gb300.workloads import (DECODE_WORKLOADS, PREFILL, STAGING,  # noqa: E402
                                               bf16_bits, fill_layer_pool, landscape_workload,
+                                              COMPOSITIONS, composition_workload,
                                               make_decode_batch, make_prefill_job,
                                               make_staging_job)
 
@@ -588,6 +589,33 @@ def read_probe(buf, reps=10):
     return buf.numel() * buf.element_size() * reps / (e0.elapsed_time(e1) * 1e-3) / 1e9
 
 
+def _decode_cell(w, device, steps, warmup):
+    """Back-to-back decode steps of one workload: GB/s, time and steps/s."""
+    batch = make_decode_batch(w, device=device)
+    tensors = _tensors(batch, device)
+    stream = torch.cuda.current_stream(device)
+    q, k, v, bt, cl, out, lse, ws = tensors
+    for _ in range(warmup):
+        cadkv.decode_attention(q, k, v, bt, cl, out=out, lse=lse, workspace=ws, stream=stream)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):   # back to back: the planner/attention overlap is kept
+        cadkv.decode_attention(q, k, v, bt, cl, out=out, lse=lse, workspace=ws, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    step_ms = e0.elapsed_time(e1) / steps
+    nbytes = decode_bytes(batch.context_lens, w.num_q_heads, w.num_kv_heads, w.head_dim)
+    cell = {"gbps": round(nbytes / (step_ms * 1e-3) / 1e9, 1),
+            "ms_per_step": round(step_ms, 4),
+            "steps_per_s": round(1e3 / step_ms, 1),
+            "tokens_per_s_per_layer": round(w.batch * 1e3 / step_ms, 1),
+            "max_context": int(batch.context_lens.max()),
+            "status": cadkv.decode_attention_status(ws)}
+    del batch, tensors
+    torch.cuda.empty_cache()
+    return cell
+
+
 def bench_landscape(device, steps, warmup, batches=(8, 32, 128, 512),
                     means=(1024, 4096, 16384, 65536), max_tokens=8 << 20):
     """Decode GB/s and steps/s over (B, mean context), 32/8 heads, D = 128."""
@@ -596,32 +624,17 @@ def bench_landscape(device, steps, warmup, batches=(8, 32, 128, 512),
         for c in means:
             if b * c > max_tokens:
                 continue
-            w = landscape_workload(b, c)
-            batch = make_decode_batch(w, device=device)
-            tensors = _tensors(batch, device)
-            stream = torch.cuda.current_stream(device)
-            q, k, v, bt, cl, out, lse, ws = tensors
-            for _ in range(warmup):
-                cadkv.decode_attention(q, k, v, bt, cl, out=out, lse=lse, workspace=ws,
-                                       stream=stream)
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            for _ in range(steps):   # back to back: the planner/attention overlap is kept
-                cadkv.decode_attention(q, k, v, bt, cl, out=out, lse=lse, workspace=ws,
-                                       stream=stream)
-            e1.record(stream)
-            torch.cuda.synchronize()
-            step_ms = e0.elapsed_time(e1) / steps
-            nbytes = decode_bytes(batch.context_lens, w.num_q_heads, w.num_kv_heads, w.head_dim)
             cells.append({"batch": b, "mean_context": c,
-                          "gbps": round(nbytes / (step_ms * 1e-3) / 1e9, 1),
-                          "ms_per_step": round(step_ms, 4),
-                          "steps_per_s": round(1e3 / step_ms, 1),
-                          "tokens_per_s_per_layer": round(b * 1e3 / step_ms, 1),
-                          "status": cadkv.decode_attention_status(tensors[7])})
-            del batch, tensors
-            torch.cuda.empty_cache()
+                          **_decode_cell(landscape_workload(b, c), device, steps, warmup)})
     return cells
+
+
+def bench_composition(device, steps, warmup, batches=(32, 128), mean=4096):
+    """Decode GB/s at a fixed batch size and mean context for five within-batch
+    length compositions (equal ... one trajectory holding half the tokens)."""
+    return [{"batch": b, "mean_context": mean, "composition": comp,
+             **_decode_cell(composition_workload(b, mean, comp), device, steps, warmup)}
+            for b in batches for comp in COMPOSITIONS]
 
 
 def bench_prefill(device, steps, warmup, cpu_baseline=False):
@@ -752,10 +765,12 @@ def main():
         return
     if args.workload == "landscape":
         cells = bench_landscape(device, args.steps, args.warmup)
+        comp = bench_composition(device, args.steps, args.warmup)
         if rank == 0:
             print(json.dumps({"workload": "decode-throughput landscape over (B, mean context), "
-                                          "32/8 heads, D=128, lengths U[C/2, 3C/2]",
-                              "unit": "GB/s", "cells": cells}), flush=True)
+                                          "32/8 heads, D=128, lengths U[C/2, 3C/2]; and over the "
+                                          "within-batch length composition at fixed (B, mean context)",
+                              "unit": "GB/s", "cells": cells, "composition_cells": comp}), flush=True)
         return
     w = DECODE_WORKLOADS[args.workload]
     batch = make_decode_batch(w, device=device, seed=w.seed + rank)

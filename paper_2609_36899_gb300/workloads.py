@@ -105,6 +105,59 @@ def landscape_workload(batch: int, mean_len: int, seed: int = 20266) -> DecodeWo
                           (lo, hi), hi, seed + batch * 1000003 + mean_len)
 
 
+COMPOSITIONS = ("equal", "uniform", "lognormal", "bimodal", "one_giant")
+
+
+def composition_lengths(batch: int, mean_len: int, composition: str,
+                        seed: int = 20269) -> np.ndarray:
+    """Context lengths of one resident batch with B * C tokens in total, spread in
+    one of five ways (the within-batch composition of the paper's Fig. 4(b)):
+
+    * ``equal``: every trajectory at C;
+    * ``uniform``: U[C/2, 3C/2];
+    * ``lognormal``: e^{N(0, 1)} rescaled to mean C (heavy-tailed, like response
+      lengths);
+    * ``bimodal``: one trajectory in 8 holds 9/16 of the tokens (4.5 C each when
+      8 divides B), the rest share the other 7/16 (C/2 each);
+    * ``one_giant``: one trajectory holds half of all tokens, the others share
+      the rest equally.
+
+    Lengths are at least 16; the total is B * C up to rounding (in expectation for
+    ``uniform``).
+    """
+    if batch < 1 or mean_len < 16:
+        raise ValueError("need batch >= 1 and mean length >= 16")
+    total = batch * mean_len
+    rng = np.random.Generator(np.random.PCG64(seed + batch * 1000003 + mean_len))
+    if composition == "equal":
+        x = np.full(batch, float(mean_len))
+    elif composition == "uniform":
+        x = rng.integers(mean_len // 2, (3 * mean_len) // 2, size=batch, endpoint=True).astype(float)
+    elif composition == "lognormal":
+        x = np.exp(rng.normal(0.0, 1.0, size=batch))
+        x *= total / x.sum()
+    elif composition == "bimodal":
+        k = max(1, batch // 8)  # long trajectories, holding 9/16 of the tokens
+        x = np.full(batch, total * 7 / 16 / max(batch - k, 1))
+        x[rng.permutation(batch)[:k]] = total * 9 / 16 / k if batch > k else total / batch
+    elif composition == "one_giant":
+        x = np.full(batch, total / 2 / max(batch - 1, 1))
+        x[rng.integers(batch)] = total / 2 if batch > 1 else total
+    else:
+        raise ValueError(f"unknown composition {composition!r}")
+    return np.maximum(np.round(x), 16).astype(np.int32)
+
+
+def composition_workload(batch: int, mean_len: int, composition: str,
+                         seed: int = 20269) -> DecodeWorkload:
+    """A decode batch (32 query / 8 KV heads, head_dim 128) with the lengths of
+    ``composition_lengths``."""
+    lens = composition_lengths(batch, mean_len, composition, seed)
+    max_len = -(-int(lens.max()) // PAGE_SIZE) * PAGE_SIZE
+    return DecodeWorkload(f"composition {composition} B={batch} C={mean_len}", batch, 32, 8, 128,
+                          "fixed", tuple(int(n) for n in lens), max_len, seed + 7 * batch + mean_len)
+
+
 def draw_lengths(kind: str, args: tuple, batch: int,
                  rng: np.random.Generator) -> np.ndarray:
     """Context lengths n_b (int32)."""

@@ -251,6 +251,28 @@ def test_landscape_cells_sampled(b, c):
     assert_close(out[idx], lse[idx], ref, ref_lse, w.name)
 
 
+@pytest.mark.parametrize("comp", ["equal", "lognormal", "bimodal", "one_giant"])
+def test_composition_cells_sampled(comp):
+    """The within-batch composition sweep at B = 128, mean 4096 (full size as
+    benched): the longest trajectory (half of all tokens for one_giant), the
+    shortest and one in the middle against the oracle."""
+    from paper_2609_36899_gb300.workloads import composition_workload
+    w = composition_workload(128, 4096, comp)
+    batch = make_decode_batch(w, device="cuda")
+    tensors = (batch.q, batch.k_pages, batch.v_pages,
+               torch.from_numpy(batch.block_table).cuda(),
+               torch.from_numpy(batch.context_lens).cuda())
+    out, lse = gpu_decode(batch, tensors=tensors)
+    assert torch.isfinite(out.float()).all() and torch.isfinite(lse).all()
+    lens = batch.context_lens
+    sample = sorted({int(np.argmax(lens)), int(np.argmin(lens)), len(lens) // 2})
+    ref, ref_lse = sampled_oracle(batch, sample)
+    idx = torch.tensor(sample, device="cuda")
+    assert_close(out[idx], lse[idx], ref, ref_lse, w.name)
+    del batch, tensors
+    torch.cuda.empty_cache()
+
+
 def test_hbm_read_probe_reads_every_word():
     g = torch.Generator().manual_seed(1)
     host = torch.randint(-2**31, 2**31 - 1, (1 << 20,), generator=g, dtype=torch.int64)
