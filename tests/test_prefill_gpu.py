@@ -174,3 +174,36 @@ def test_prefill_rejects_chunk_longer_than_context():
         bf16_bits(q[:5]), offs[:2], bf16_bits(batch.k_pages), bf16_bits(batch.v_pages),
         batch.block_table[:1], batch.context_lens[:1])
     assert_close(out[:5], None, ref, ref_lse, "trajectory 0")
+
+
+def test_prefill_zero_length_chunks_and_no_lse():
+    """Trajectories that re-prefill nothing sit between ones that do; their rows
+    do not exist, and the others are unaffected.  lse may be left out."""
+    lens, chunks = [300, 50, 700, 129], [0, 50, 0, 129]
+    batch, offs, q = _case(lens, chunks, 8, 2, seed=480)
+    out, lse, ws = cadkv.prefill_attention(
+        q.cuda(), torch.from_numpy(offs).cuda(), batch.k_pages.cuda(), batch.v_pages.cuda(),
+        torch.from_numpy(batch.block_table).cuda(), torch.from_numpy(batch.context_lens).cuda(),
+        want_lse=False)
+    torch.cuda.synchronize()
+    assert lse is None and cadkv.prefill_attention_status(ws) == 0
+    ref, ref_lse = _oracle(batch, offs, q)
+    assert_close(out, None, ref, ref_lse, "prefill with empty chunks, no lse")
+
+
+def test_prefill_empty_job():
+    batch, offs, q = _case([40, 60], [0, 0], 4, 1, seed=485)
+    out, lse, ws = _run(batch, offs, q)
+    assert out.shape[0] == 0 and cadkv.prefill_attention_status(ws) == 0
+
+
+def test_prefill_repeat_calls_bit_identical():
+    """Split items merge their pieces in piece order, whichever CTA finishes
+    last: two calls give the same bits."""
+    lens, chunks = [20000, 9000], [64, 300]
+    batch, offs, q = _case(lens, chunks, 8, 2, seed=490)
+    a_out, a_lse, _ = _run(batch, offs, q)
+    b_out, b_lse, _ = _run(batch, offs, q)
+    assert torch.equal(a_out, b_out) and torch.equal(a_lse, b_lse)
+    ref, ref_lse = _oracle(batch, offs, q)
+    assert_close(a_out, a_lse, ref, ref_lse, "prefill repeat")
