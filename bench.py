@@ -14,7 +14,7 @@ kernel's roofline fraction, an end-to-end number through the C ABI with
 host buffers, the fp64 CPU oracle timed on a bounded sample, SM clocks
 during the timed region and, as a secondary measurement, prefix staging.
 
-``--impl reference`` times the oracle (the CPU reference of this build) on
+``--impl reference`` times the oracle (the library's fp64 CPU reference) on
 the same workload and prints the same metric.
 Multi-GPU (torchrun): each rank runs its own batch (weak scaling, no
 collective on the data path); rank 0 prints the whole-job numbers.
