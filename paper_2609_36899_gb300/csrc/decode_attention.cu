@@ -27,7 +27,9 @@
 //    A trajectory-head that lies inside one slice is written straight to
 //    `out`; otherwise the slice writes a partial (o, log2-sum-exp) and the CTA
 //    that delivers a unit's last partial merges all of them in slice order
-//    (deterministic), so no separate merge kernel runs.
+//    (deterministic), so no separate merge kernel runs.  One release/acquire
+//    atomic per partial orders the partials; its result is read only after the
+//    CTA's next segment, so the warps do not stall on it.
 //  * Every wait is bounded (kWaitLimitNs); on timeout the kernel records
 //    CADKV_ERR_TIMEOUT, drains its own copies and returns.
 #include <cfloat>
@@ -477,6 +479,58 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     const int ct = tid;                             // consumer thread 0..127
     uint32_t k = 0, sc = 0, cphase = 0;
     bool ok = true;
+    SegDesc pd{};         // the last partial whose unit may still need its merge
+    bool pending = false;
+    int pend_old = 0;     // thread 0: the unit counter before pd's partial was counted
+    // The CTA that completes a unit merges its partials in slice order.
+    auto merge_unit = [&](const SegDesc &u) {
+        const int slot0 = u.unit + u.first;
+        for (int it = ct; it < G * (D / 8); it += kNumConsumerWarps * 32) {
+            const int h = it / (D / 8), d0 = (it % (D / 8)) * 8;
+            // One pass in slice order, rescaling the running sum as the max grows.
+            float M = -INFINITY, L = 0.f;
+            float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+            for (int s2 = 0; s2 < u.count; ++s2) {
+                const size_t sl = (size_t)(slot0 + s2);
+                const float lse_s = __ldcg(p.part_lse + sl * G + h);
+                const float4 *src = reinterpret_cast<const float4 *>(p.part_o + (sl * G + h) * D + d0);
+                const float4 u0 = __ldcg(src), u1 = __ldcg(src + 1);
+                const float Mn = fmaxf(M, lse_s);
+                const float a = exp2_approx(M - Mn), w = exp2_approx(lse_s - Mn);
+                M = Mn;
+                L = L * a + w;
+                acc[0] = acc[0] * a + w * u0.x;
+                acc[1] = acc[1] * a + w * u0.y;
+                acc[2] = acc[2] * a + w * u0.z;
+                acc[3] = acc[3] * a + w * u0.w;
+                acc[4] = acc[4] * a + w * u1.x;
+                acc[5] = acc[5] * a + w * u1.y;
+                acc[6] = acc[6] * a + w * u1.z;
+                acc[7] = acc[7] * a + w * u1.w;
+            }
+            const float inv = 1.f / L;
+            uint4 packed;
+            packed.x = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+            packed.y = pack_bf16x2(acc[2] * inv, acc[3] * inv);
+            packed.z = pack_bf16x2(acc[4] * inv, acc[5] * inv);
+            packed.w = pack_bf16x2(acc[6] * inv, acc[7] * inv);
+            const size_t row = (size_t)u.b * p.num_q_heads + u.kvh * G + h;
+            *reinterpret_cast<uint4 *>(p.out + row * D + d0) = packed;
+            if (d0 == 0 && p.lse)
+                p.lse[row] = (M + __log2f(L)) * kLn2;
+        }
+    };
+    auto resolve_pending = [&]() -> bool {
+        if (ct == 0)
+            *is_last_flag = (pend_old == pd.count - 1) ? 1 : 0;
+        if (!consumer_sync(cons_bar, cphase, abort_flag))
+            return false;
+        if (*is_last_flag)
+            merge_unit(pd);
+        pending = false;
+        return true;
+    };
 
     for (;;) {
         const uint32_t r = sc % kSegRing;
@@ -672,62 +726,32 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     p.part_lse[(size_t)d.slot * G + h] = lse2;
             }
         }
-        if (partial)
-            __threadfence();
         ok = consumer_sync(cons_bar, cphase, abort_flag);
         if (!ok)
             break;
+        // the previous partial's counter update has long completed: merge its
+        // unit now if this CTA delivered that unit's last partial
+        if (pending) {
+            ok = resolve_pending();
+            if (!ok)
+                break;
+        }
         if (!partial)
             continue;
 
-        // ---- the CTA that completes a unit merges its partials in slice order
+        // ---- count this partial; whether it completes the unit is read after
+        // the next segment (or at the end), so the warps go straight on to it
         if (ct == 0) {
-            const int old = atomicAdd(&p.unit_counter[d.unit], 1);
-            *is_last_flag = (old == d.count - 1) ? 1 : 0;
+            // acq_rel at GPU scope: releases this CTA's partial stores (ordered
+            // before it by the barrier above) and acquires every earlier slice's
+            asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], 1;"
+                         : "=r"(pend_old) : "l"(&p.unit_counter[d.unit]) : "memory");
         }
-        ok = consumer_sync(cons_bar, cphase, abort_flag);
-        if (!ok)
-            break;
-        if (*is_last_flag) {
-            __threadfence();
-            const int slot0 = d.unit + d.first;
-            for (int it = ct; it < G * (D / 8); it += kNumConsumerWarps * 32) {
-                const int h = it / (D / 8), d0 = (it % (D / 8)) * 8;
-                // One pass in slice order, rescaling the running sum as the max grows.
-                float M = -INFINITY, L = 0.f;
-                float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-#pragma unroll 4
-                for (int s2 = 0; s2 < d.count; ++s2) {
-                    const size_t sl = (size_t)(slot0 + s2);
-                    const float lse_s = __ldcg(p.part_lse + sl * G + h);
-                    const float4 *src = reinterpret_cast<const float4 *>(p.part_o + (sl * G + h) * D + d0);
-                    const float4 u0 = __ldcg(src), u1 = __ldcg(src + 1);
-                    const float Mn = fmaxf(M, lse_s);
-                    const float a = exp2_approx(M - Mn), w = exp2_approx(lse_s - Mn);
-                    M = Mn;
-                    L = L * a + w;
-                    acc[0] = acc[0] * a + w * u0.x;
-                    acc[1] = acc[1] * a + w * u0.y;
-                    acc[2] = acc[2] * a + w * u0.z;
-                    acc[3] = acc[3] * a + w * u0.w;
-                    acc[4] = acc[4] * a + w * u1.x;
-                    acc[5] = acc[5] * a + w * u1.y;
-                    acc[6] = acc[6] * a + w * u1.z;
-                    acc[7] = acc[7] * a + w * u1.w;
-                }
-                const float inv = 1.f / L;
-                uint4 packed;
-                packed.x = pack_bf16x2(acc[0] * inv, acc[1] * inv);
-                packed.y = pack_bf16x2(acc[2] * inv, acc[3] * inv);
-                packed.z = pack_bf16x2(acc[4] * inv, acc[5] * inv);
-                packed.w = pack_bf16x2(acc[6] * inv, acc[7] * inv);
-                const size_t row = (size_t)d.b * p.num_q_heads + q_head0 + h;
-                *reinterpret_cast<uint4 *>(p.out + row * D + d0) = packed;
-                if (d0 == 0 && p.lse)
-                    p.lse[row] = (M + __log2f(L)) * kLn2;
-            }
-        }
+        pd = d;
+        pending = true;
     }
+    if (ok && pending)
+        ok = resolve_pending();
     if (!ok && lane == 0) {
         *abort_flag = 1;
         record_status(&p.hdr->status, CADKV_ERR_TIMEOUT);
