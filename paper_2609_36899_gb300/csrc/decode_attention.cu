@@ -254,6 +254,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     using C = AttnConfig<D>;
     constexpr int S = C::kStages;
     static_assert(kIssueGroup <= S, "a parallel issue group must not reuse a stage");
+    // Page i of a segment goes to consumer warp i % kNumConsumerWarps and lands in
+    // stage (k + i) % S.  With S a multiple of the warp count, the next use of a
+    // stage within a segment belongs to the warp that released its last use, so
+    // no warp can wait on a stage two phases ahead, where a parity wait would
+    // match the stale phase (the end-of-segment barrier covers segment borders).
+    static_assert(S % kNumConsumerWarps == 0, "each stage must be reused by the warp that released it");
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(align_up(reinterpret_cast<size_t>(smem_raw), 1024));
     uint8_t *stages = smem + C::kStagesOff;
