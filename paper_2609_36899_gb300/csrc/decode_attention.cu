@@ -19,7 +19,8 @@
 //    guarded by mbarriers, plus a 1-D bulk copy of the G query rows of every
 //    new segment.  Each KV page is read from HBM exactly once per KV head:
 //    all G query heads of the group share it (grouped-query attention).
-//  * Four consumer warps take pages round-robin.  Per page a warp computes
+//  * Eight consumer warps take pages round-robin (four could not keep up
+//    with HBM on every SM).  Per page a warp computes
 //    S^T = K Q^T with mma.sync m16n8k16 (16 tokens x 8 query heads), runs the
 //    online softmax in registers (warp shuffles for the per-head max), turns
 //    P^T into the B operand with movmatrix, and accumulates O^T += V^T P^T.
@@ -188,7 +189,7 @@ struct SegDesc {
 
 template <int D>
 struct AttnConfig {
-    static constexpr int kStages = D == 128 ? 20 : 28;
+    static constexpr int kStages = D == 128 ? 16 : 32;
     static constexpr int kBoxes = D / 64;                    // 64-element (128 B) TMA boxes per row
     static constexpr int kBoxBytes = kPageSize * 128;        // 16 rows x 128 B
     static constexpr int kKBytes = kBoxes * kBoxBytes;       // one page-head of K
@@ -569,8 +570,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
 
         const int npg = d.num_pages;
-        // Page i of a segment always goes to warp i % 4, whatever the CTA did
-        // before, so the summation order (and the result) is deterministic.
+        // Page i of a segment always goes to warp i % kNumConsumerWarps, whatever
+        // the CTA did before, so the summation order (and the result) is
+        // deterministic.
         for (int i = warp; i < npg; i += kNumConsumerWarps) {
             const uint32_t kk_idx = k + i;
             const uint32_t st = kk_idx % S;

@@ -13,7 +13,7 @@ namespace cadkv {
 
 constexpr int kPageSize = 16;      // tokens per KV page
 constexpr int kMaxGroup = 8;       // query heads per KV head handled by one tile
-constexpr int kNumConsumerWarps = 4;
+constexpr int kNumConsumerWarps = 8;
 constexpr int kAttnThreads = (kNumConsumerWarps + 1) * 32;
 constexpr int kSegRing = 8;        // segment descriptors in flight per CTA
 constexpr int kSlicesPerCta = 4;   // dynamic work slices per persistent CTA
