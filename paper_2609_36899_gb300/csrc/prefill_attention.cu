@@ -22,7 +22,7 @@
 //    and hands them to the other warps through a small ring; every ring and
 //    barrier phase counts the CTA's key tiles or units, so the pipelines run
 //    on from one unit to the next.
-//  * Warp 10 loads each segment's two Q tiles (3-D tensor map, two 64-column
+//  * Warp 2 loads each segment's two Q tiles (3-D tensor map, two 64-column
 //    panels each, 128-byte swizzle) once the previous segment's S MMAs are
 //    done.  Warp 0 streams K and V tiles of 128 keys (8 pages, two 2 KB boxes
 //    per page and operand, issued from 32 lanes at once) into a 3-stage K ring
@@ -34,13 +34,16 @@
 //    from TMEM (the MMA form whose A operand lives in tensor memory) and V as
 //    an MN-major operand from the swizzled stage.  Tiles A and B alternate, so
 //    the tensor cores work on one tile while the softmax works on the other.
-//  * Warps 2-5 (tile A) and 6-9 (tile B): one query row per thread = one TMEM
-//    lane.  The row's 128 scores come in one burst of tcgen05.ld, causal mask
-//    only on tiles that cross the diagonal, running max with lazy O rescaling
-//    (only when the max grows by more than 2^8; the decision is warp-uniform
-//    since tcgen05.ld/st are warp-collective), P = 2^(s - m) packed to bf16
-//    and stored with tcgen05.st over the S columns already consumed.  At the
-//    end of a segment: O / l and lse, or the piece's partial row.
+//  * Warps 4-7 (tile A) and 8-11 (tile B): one query row per thread = one TMEM
+//    lane (setmaxnreg gives them 192 registers, the control warps 120).  The
+//    row's 128 scores come in one burst of tcgen05.ld, causal mask only on
+//    tiles that cross the diagonal.  P = 2^(s - m) is taken against the running
+//    max m without a max pass while every P stays below 2^8 (the tile's row sum
+//    bounds them); otherwise, and on a row's first tile, the max is taken, m
+//    moves and O is rescaled in TMEM (warp-uniform decisions, since tcgen05.ld/st
+//    are warp-collective).  P is packed to bf16 and stored with tcgen05.st over
+//    the S columns already consumed.  At the end of a segment: O / l and lse,
+//    or the piece's partial row.
 //  * All waits are bounded; on timeout the kernel records CADKV_ERR_TIMEOUT,
 //    waits for its own copies and MMAs, frees TMEM and returns.
 #include <cfloat>
