@@ -770,15 +770,11 @@ template <int D>
 cudaError_t launch_attention_d(const AttnParams &p, const CUtensorMap &kmap,
                                const CUtensorMap &vmap, int grid, cudaStream_t stream)
 {
-    static bool configured = false;
+    static std::atomic<uint64_t> configured{0};
     const size_t smem = AttnConfig<D>::kBytes;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_attention_kernel<D>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess)
-            return e;
-        configured = true;
-    }
+    cudaError_t e = ensure_smem_limit(decode_attention_kernel<D>, (int)smem, configured);
+    if (e != cudaSuccess)
+        return e;
     // Programmatic dependent launch: may start while the planner still runs.
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(grid);

@@ -1,6 +1,7 @@
 // internal.h -- types shared by the host launchers and the kernels.
 #pragma once
 
+#include <atomic>
 #include <cstddef>
 #include <cstdint>
 #include <cuda.h>
@@ -10,6 +11,27 @@
 #include "cadkv.h"
 
 namespace cadkv {
+
+// Raises a kernel's dynamic shared-memory limit to `bytes`, once per device:
+// the attribute belongs to the device's context, and host threads may launch
+// concurrently.  `done` keeps one bit per device id below 64.
+template <typename Kernel>
+inline cudaError_t ensure_smem_limit(Kernel *kernel, int bytes, std::atomic<uint64_t> &done)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess)
+        return e;
+    const uint64_t bit = dev >= 0 && dev < 64 ? 1ull << dev : 0;
+    if (bit && (done.load(std::memory_order_acquire) & bit))
+        return cudaSuccess;
+    e = cudaFuncSetAttribute(reinterpret_cast<const void *>(kernel),
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess && bit)
+        done.fetch_or(bit, std::memory_order_release);
+    return e;
+}
+
 
 constexpr int kPageSize = 16;      // tokens per KV page
 constexpr int kMaxGroup = 8;       // query heads per KV head handled by one tile

@@ -1025,17 +1025,13 @@ size_t prefill_smem_bytes() { return sizeof(PrefillSmem) + 1024; }
 cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, const CUtensorMap &kmap,
                            const CUtensorMap &vmap, cudaStream_t stream)
 {
-    static bool configured = false;
+    static std::atomic<uint64_t> configured{0};
     const size_t smem = prefill_smem_bytes();
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(prefill_attention_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess)
-            return e;
-        configured = true;
-    }
+    cudaError_t e = ensure_smem_limit(prefill_attention_kernel, (int)smem, configured);
+    if (e != cudaSuccess)
+        return e;
     prefill_plan_kernel<<<1, 1024, 0, stream>>>(p);
-    cudaError_t e = cudaGetLastError();
+    e = cudaGetLastError();
     if (e != cudaSuccess)
         return e;
     // Programmatic dependent launch: the attention kernel's prologue overlaps the planner.
