@@ -635,10 +635,12 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return CADKV_ERR_CUDA;
     }
-    int whole = 0;  // the prefill kernel uses 2-D boxes of one 64-column panel
-    if (encode_pages_map(&kmap, k_pages, num_pages, num_kv_heads, head_dim, false, &whole) !=
+    // K: 2-D boxes of one 64-column panel (its operand is panel-major); V: whole
+    // 4 KB (page, head) blocks when the driver accepts the 4-D view
+    int k_whole = 0, v_whole = 0;
+    if (encode_pages_map(&kmap, k_pages, num_pages, num_kv_heads, head_dim, false, &k_whole) !=
             CADKV_OK ||
-        encode_pages_map(&vmap, v_pages, num_pages, num_kv_heads, head_dim, false, &whole) !=
+        encode_pages_map(&vmap, v_pages, num_pages, num_kv_heads, head_dim, true, &v_whole) !=
             CADKV_OK)
         return CADKV_ERR_CUDA;
     const int ctas = prefill_ctas();
@@ -663,6 +665,7 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
     p.group = group;
     p.max_pages = max_pages;
     p.num_pages = num_pages;
+    p.v_whole = v_whole;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
     return launch_prefill(p, qmap, kmap, vmap, reinterpret_cast<cudaStream_t>(stream)) ==
                    cudaSuccess

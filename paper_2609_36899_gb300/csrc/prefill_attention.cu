@@ -24,10 +24,14 @@
 //    on from one unit to the next.
 //  * Warp 2 loads each segment's two Q tiles (3-D tensor map, two 64-column
 //    panels each, 128-byte swizzle) once the previous segment's S MMAs are
-//    done.  Warp 0 streams K and V tiles of 128 keys (8 pages, two 2 KB boxes
-//    per page and operand, issued from 32 lanes at once) into a 3-stage K ring
-//    and a 2-stage V ring; K is released as soon as both S MMAs have read it,
-//    so it is loaded a tile ahead of V.
+//    done.  Warp 0 streams K and V tiles of 128 keys (8 pages, issued from 32
+//    lanes at once) into a 3-stage K ring and a 2-stage V ring; K is released
+//    as soon as both S MMAs have read it, so it is loaded a tile ahead of V.
+//    The TMA unit's rate per box bounds this kernel (a 2 KB box costs about as
+//    long as a 4 KB one), so V comes as one 4 KB box per (page, KV head)
+//    block, landing page-major, which its MN-major operand descriptor allows;
+//    K's K-major operand needs all 128 keys of a 64-column panel at one
+//    stride, so it keeps two 2 KB boxes per page.
 //  * Warp 1 (MMA issuer, one lane) keeps S_A, S_B, O_A, O_B in TMEM (4 x 128
 //    fp32 columns).  Per key tile j it issues S_X = Q_X K_j^T and, once the
 //    softmax has turned S_X into P_X, O_X += P_X V_j with P_X read straight
@@ -541,16 +545,23 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                     break;
                 const int kt = op == 0 ? ktk : ktv;
                 const int pages = op == 0 ? pages_k : pages_v;
-                if ((op == 0 ? do_k : do_v) && pg < pages) {
+                // V as whole 4 KB (page, head) blocks when the 4-D view exists: one box
+                // per page (lane hh == 0), landing page-major ([page][half][16][128 B])
+                if ((op == 0 ? do_k : do_v) && pg < pages && (op == 0 || !p.v_whole || hh == 0)) {
                     int phys = p.block_table[(size_t)sg.b * p.max_pages + kt * (kKeys / kPageSize) + pg];
                     if (phys < 0 || phys >= p.num_pages) {
                         record_status(&p.hdr->status, CADKV_ERR_OOB);
                         phys = 0;
                     }
                     const int y = (phys * p.num_kv_heads + sg.g) * kPageSize;
-                    uint8_t *dst = (op == 0 ? sm.k[sk] : sm.v[sv]) + hh * kPanel + pg * 2048;
-                    tma_load_2d(dst, op == 0 ? &kmap : &vmap, hh * 64, y,
-                                op == 0 ? &sm.k_full[sk] : &sm.v_full[sv], policy);
+                    if (op == 1 && p.v_whole) {
+                        tma_load_4d(sm.v[sv] + pg * kPageBlock, &vmap, 0, 0, 0, phys * p.num_kv_heads + sg.g,
+                                    &sm.v_full[sv], policy);
+                    } else {
+                        uint8_t *dst = (op == 0 ? sm.k[sk] : sm.v[sv]) + hh * kPanel + pg * 2048;
+                        tma_load_2d(dst, op == 0 ? &kmap : &vmap, hh * 64, y,
+                                    op == 0 ? &sm.k_full[sk] : &sm.v_full[sv], policy);
+                    }
                 }
                 nk += do_k;
                 nv += do_v;
@@ -626,7 +637,11 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             }
 #pragma unroll
             for (int k = 0; k < kKeys / 16; ++k)
-                v_lo[0][k] = (uint32_t)desc_sw128(smem_addr(sm.v[0] + k * 2048), kPanel, 1024);
+                // keys 16k .. 16k+15: page k.  Page-major V: its two D halves 2 KB apart;
+                // panel-major V: 2 KB into each 16 KB panel
+                v_lo[0][k] = p.v_whole
+                                 ? (uint32_t)desc_sw128(smem_addr(sm.v[0] + k * kPageBlock), 2048, 1024)
+                                 : (uint32_t)desc_sw128(smem_addr(sm.v[0] + k * 2048), kPanel, 1024);
             if (lane == 0) {
             auto desc = [&](uint32_t lo_word) { return ((uint64_t)d_hi << 32) | lo_word; };
             constexpr uint32_t kStage16 = kTileBytes >> 4;  // one ring stage in descriptor units
@@ -867,7 +882,9 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                         break;
                     if (key0 + row > sg.pos_max) {
                         for (int h = 0; h < 2; ++h) {
-                            uint4 *rz = reinterpret_cast<uint4 *>(sm.v[sv] + h * kPanel + row * 128);
+                            uint4 *rz = reinterpret_cast<uint4 *>(
+                                p.v_whole ? sm.v[sv] + (row >> 4) * kPageBlock + h * 2048 + (row & 15) * 128
+                                          : sm.v[sv] + h * kPanel + row * 128);
 #pragma unroll
                             for (int c16 = 0; c16 < 8; ++c16)
                                 rz[c16] = make_uint4(0, 0, 0, 0);
