@@ -27,8 +27,8 @@
 //    done.  Warp 0 streams K and V tiles of 128 keys (8 pages, issued from 32
 //    lanes at once) into a 3-stage K ring and a 2-stage V ring; K is released
 //    as soon as both S MMAs have read it, so it is loaded a tile ahead of V.
-//    The TMA unit's rate per box bounds this kernel (a 2 KB box costs about as
-//    long as a 4 KB one), so V comes as one 4 KB box per (page, KV head)
+//    The SM's TMA box rate bounds this kernel (~98 cycles per swizzled 2 KB box,
+//    ~144 per 4 KB box, measured), so V comes as one 4 KB box per (page, KV head)
 //    block, landing page-major, which its MN-major operand descriptor allows;
 //    K's K-major operand needs all 128 keys of a 64-column panel at one
 //    stride, so it keeps two 2 KB boxes per page.
