@@ -239,7 +239,10 @@ size_t prefill_attention_workspace_size(int batch);
  * order, by the CTA that completes the item.  The workspace must not be used
  * by two calls in flight at once.
  * Supported: head_dim 128, page_size 16, G = Hq / Hkv in 1..8 (the Qwen3
- * models of Sec. 6 have G = 4, 5 and 8).
+ * models of Sec. 6 have G = 4, 5 and 8); anything else returns
+ * CADKV_ERR_UNSUPPORTED, as does a driver that cannot describe V as whole
+ * 4 KB (page, KV head) blocks (a 4-D tensor map: V is loaded one block per
+ * TMA box).
  * A trajectory with C_b > n_b or n_b out of range is skipped (its rows are
  * not written) and CADKV_ERR_SHAPE lands in the status word.
  */

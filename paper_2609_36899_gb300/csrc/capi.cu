@@ -636,13 +636,15 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
             return CADKV_ERR_CUDA;
     }
     // K: 2-D boxes of one 64-column panel (its operand is panel-major); V: whole
-    // 4 KB (page, head) blocks when the driver accepts the 4-D view
+    // 4 KB (page, head) blocks through the 4-D view, which the kernel requires
     int k_whole = 0, v_whole = 0;
     if (encode_pages_map(&kmap, k_pages, num_pages, num_kv_heads, head_dim, false, &k_whole) !=
             CADKV_OK ||
         encode_pages_map(&vmap, v_pages, num_pages, num_kv_heads, head_dim, true, &v_whole) !=
             CADKV_OK)
         return CADKV_ERR_CUDA;
+    if (!v_whole)
+        return CADKV_ERR_UNSUPPORTED;
     const int ctas = prefill_ctas();
     const PrefillWorkspaceLayout L = prefill_workspace_layout(batch, ctas);
     uint8_t *ws = static_cast<uint8_t *>(workspace);
@@ -665,7 +667,6 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
     p.group = group;
     p.max_pages = max_pages;
     p.num_pages = num_pages;
-    p.v_whole = v_whole;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
     return launch_prefill(p, qmap, kmap, vmap, reinterpret_cast<cudaStream_t>(stream)) ==
                    cudaSuccess

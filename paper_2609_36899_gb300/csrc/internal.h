@@ -128,7 +128,6 @@ struct PrefillParams {
     float *partial_o;            // [2 * num_ctas][128][256] O / l of a piece's rows, column-major
     long long total_q;           // rows of q / out; offsets beyond it are rejected
     int batch, num_q_heads, num_kv_heads, group, max_pages, num_pages, num_ctas;
-    int v_whole;                 // 1: V loaded as whole 4 KB (page, head) blocks, page-major
     float scale_log2;
 };
 

@@ -545,23 +545,21 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                     break;
                 const int kt = op == 0 ? ktk : ktv;
                 const int pages = op == 0 ? pages_k : pages_v;
-                // V as whole 4 KB (page, head) blocks when the 4-D view exists: one box
-                // per page (lane hh == 0), landing page-major ([page][half][16][128 B])
-                if ((op == 0 ? do_k : do_v) && pg < pages && (op == 0 || !p.v_whole || hh == 0)) {
+                // V as whole 4 KB (page, head) blocks: one box per page (lane hh == 0),
+                // landing page-major ([page][half][16][128 B])
+                if ((op == 0 ? do_k : do_v) && pg < pages && (op == 0 || hh == 0)) {
                     int phys = p.block_table[(size_t)sg.b * p.max_pages + kt * (kKeys / kPageSize) + pg];
                     if (phys < 0 || phys >= p.num_pages) {
                         record_status(&p.hdr->status, CADKV_ERR_OOB);
                         phys = 0;
                     }
                     const int y = (phys * p.num_kv_heads + sg.g) * kPageSize;
-                    if (op == 1 && p.v_whole) {
+                    if (op == 1)
                         tma_load_4d(sm.v[sv] + pg * kPageBlock, &vmap, 0, 0, 0, phys * p.num_kv_heads + sg.g,
                                     &sm.v_full[sv], policy);
-                    } else {
-                        uint8_t *dst = (op == 0 ? sm.k[sk] : sm.v[sv]) + hh * kPanel + pg * 2048;
-                        tma_load_2d(dst, op == 0 ? &kmap : &vmap, hh * 64, y,
-                                    op == 0 ? &sm.k_full[sk] : &sm.v_full[sv], policy);
-                    }
+                    else
+                        tma_load_2d(sm.k[sk] + hh * kPanel + pg * 2048, &kmap, hh * 64, y, &sm.k_full[sk],
+                                    policy);
                 }
                 nk += do_k;
                 nv += do_v;
@@ -637,11 +635,9 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
             }
 #pragma unroll
             for (int k = 0; k < kKeys / 16; ++k)
-                // keys 16k .. 16k+15: page k.  Page-major V: its two D halves 2 KB apart;
-                // panel-major V: 2 KB into each 16 KB panel
-                v_lo[0][k] = p.v_whole
-                                 ? (uint32_t)desc_sw128(smem_addr(sm.v[0] + k * kPageBlock), 2048, 1024)
-                                 : (uint32_t)desc_sw128(smem_addr(sm.v[0] + k * 2048), kPanel, 1024);
+                // keys 16k .. 16k+15 = page k of the page-major V stage: its two
+                // 64-column halves are 2 KB apart (LBO), 8-key groups 1 KB (SBO)
+                v_lo[0][k] = (uint32_t)desc_sw128(smem_addr(sm.v[0] + k * kPageBlock), 2048, 1024);
             if (lane == 0) {
             auto desc = [&](uint32_t lo_word) { return ((uint64_t)d_hi << 32) | lo_word; };
             constexpr uint32_t kStage16 = kTileBytes >> 4;  // one ring stage in descriptor units
@@ -882,9 +878,8 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                         break;
                     if (key0 + row > sg.pos_max) {
                         for (int h = 0; h < 2; ++h) {
-                            uint4 *rz = reinterpret_cast<uint4 *>(
-                                p.v_whole ? sm.v[sv] + (row >> 4) * kPageBlock + h * 2048 + (row & 15) * 128
-                                          : sm.v[sv] + h * kPanel + row * 128);
+                            uint4 *rz = reinterpret_cast<uint4 *>(sm.v[sv] + (row >> 4) * kPageBlock +
+                                                                  h * 2048 + (row & 15) * 128);
 #pragma unroll
                             for (int c16 = 0; c16 < 8; ++c16)
                                 rz[c16] = make_uint4(0, 0, 0, 0);
