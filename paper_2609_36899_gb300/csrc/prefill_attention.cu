@@ -490,8 +490,9 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
         }
         // Step J of a segment issues its K_J (lanes 0-15) and V_{J-1} (lanes
         // 16-31): K is freed right after the S MMAs while V waits for PV, so each
-        // stream is gated only by its own ring and K runs a tile ahead.  Box =
-        // one 64-column panel of one page: page = (lane / 2) % 8, panel = lane % 2.
+        // stream is gated only by its own ring and K runs a tile ahead.  Page =
+        // (lane / 2) % 8; a K box is the 64-column panel lane % 2 of it, a V box
+        // the whole 4 KB block (issued by the even lane).
         const int op = lane >> 4, pg = (lane >> 1) & 7, hh = lane & 1;
         int nk = 0, nv = 0;  // K and V tiles this CTA has loaded
         for (long long k = 0; ok; ++k) {
