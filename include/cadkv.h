@@ -242,7 +242,9 @@ size_t prefill_attention_workspace_size(int batch);
  * models of Sec. 6 have G = 4, 5 and 8); anything else returns
  * CADKV_ERR_UNSUPPORTED, as does a driver that cannot describe V as whole
  * 4 KB (page, KV head) blocks (a 4-D tensor map: V is loaded one block per
- * TMA box).
+ * TMA box), or a build whose kernel was given fewer registers per thread at
+ * launch than its warp roles divide among themselves (checked once, before
+ * the first launch).
  * A trajectory with C_b > n_b or n_b out of range is skipped (its rows are
  * not written) and CADKV_ERR_SHAPE lands in the status word.
  */

@@ -645,6 +645,8 @@ int prefill_attention(const void *q, const int64_t *q_offsets, const void *k_pag
         return CADKV_ERR_CUDA;
     if (!v_whole)
         return CADKV_ERR_UNSUPPORTED;
+    if (!prefill_register_split_fits())
+        return CADKV_ERR_UNSUPPORTED;
     const int ctas = prefill_ctas();
     const PrefillWorkspaceLayout L = prefill_workspace_layout(batch, ctas);
     uint8_t *ws = static_cast<uint8_t *>(workspace);

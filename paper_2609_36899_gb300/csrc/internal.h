@@ -132,6 +132,7 @@ struct PrefillParams {
 };
 
 size_t prefill_smem_bytes();
+bool prefill_register_split_fits();  // the kernel's launch registers cover its setmaxnreg split
 cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, const CUtensorMap &kmap,
                            const CUtensorMap &vmap, cudaStream_t stream);
 

@@ -1035,6 +1035,24 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
 
 size_t prefill_smem_bytes() { return sizeof(PrefillSmem) + 1024; }
 
+// setmaxnreg.inc waits until the CTA has the registers it asks for, and it only
+// has what it was launched with: a build whose launch allocation is below the
+// split would wait forever, so it is refused before launch.
+bool prefill_register_split_fits()
+{
+    static std::atomic<int> fits{-1};
+    int f = fits.load();
+    if (f < 0) {
+        cudaFuncAttributes a{};
+        f = cudaFuncGetAttributes(&a, prefill_attention_kernel) == cudaSuccess &&
+                    128 * kControlRegs + kSoftmaxThreads * kSoftmaxRegs <= kPrefillThreads * a.numRegs
+                ? 1
+                : 0;
+        fits.store(f);
+    }
+    return f == 1;
+}
+
 cudaError_t launch_prefill(const PrefillParams &p, const CUtensorMap &qmap, const CUtensorMap &kmap,
                            const CUtensorMap &vmap, cudaStream_t stream)
 {
