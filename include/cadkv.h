@@ -125,7 +125,10 @@ size_t decode_attention_workspace_size(int batch, int num_q_heads, int num_kv_he
                                        int head_dim, int max_pages);
 
 /*
- * One decode step of attention for `batch` trajectories (one query token each).
+ * One decode step of attention for `batch` trajectories (one query token each):
+ * the bandwidth-bound step of autoregressive rollout (Sec. 2.3, Sec. 3.1),
+ * with the attention operator and paged KV cache of the paper's inference
+ * backend (Sec. 5), as written out at the top of this file.
  *   q            bf16 [batch][num_q_heads][head_dim]
  *   k_pages      bf16 [num_pages][num_kv_heads][16][head_dim]   (one layer)
  *   v_pages      bf16 [num_pages][num_kv_heads][16][head_dim]
@@ -267,7 +270,7 @@ size_t kv_prefix_stage_workspace_size(int batch);
 
 /*
  * Gather the first n_b tokens of layers [layer_begin, layer_end) of every
- * trajectory b from the pool into contiguous rows (Sec. 5, late-bound KV
+ * trajectory b from the pool into contiguous rows (Sec. 4.4, late-bound KV
  * preparation: the departing trajectory's prefix is snapshotted):
  *   dst[off_b + (((l - layer_begin)*2 + kv)*Hkv + h)*n_b*D + t*D + d]
  *       = (kv == 0 ? K : V)_l[block_table[b][t/16]][h][t%16][d]
@@ -348,9 +351,12 @@ int cadkv_hbm_read_probe(const void *buf, size_t bytes, unsigned long long *sink
  * GPU that loads the library holds until the process exits.  Nothing is
  * allocated: no cudaMalloc, no cudaFree, no allocating library routine.
  *
- * - The first call on a device looks up that device's address of the array
- *   (cudaGetSymbolAddress, with the device current) and caches it; make that
- *   first call before any stream capture on the device.
+ * - The first call in a device's context looks up that context's address of
+ *   the array (cudaGetSymbolAddress, with the device current) and caches it
+ *   with the context's id; make that first call before any stream capture on
+ *   the device.  A call made in another context of the same device (after
+ *   cudaDeviceReset, or under a context the caller made current) looks the
+ *   address up again: a cached address is tied to its context.
  * - A problem whose scratch would exceed CADKV_NOALLOC_SCRATCH_BYTES is
  *   rejected with CADKV_ERR_WORKSPACE before anything is launched (the
  *   requirement is decode_attention_workspace_size() of the same sizes).

@@ -718,23 +718,69 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[CADKV_NOALLOC_S
 
 namespace {
 
-// Device address of g_noalloc_scratch on the current device, looked up once
-// per device and cached.
+using CtxGetCurrentFn = CUresult (*)(CUcontext *);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long *);
+
+// Process-unique id of the CUDA context current on this thread, or 0 when no
+// context is current or the driver cannot tell.
+unsigned long long current_context_id()
+{
+    static CtxGetCurrentFn get_current = nullptr;
+    static CtxGetIdFn get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *a = nullptr, *b = nullptr;
+        cudaDriverEntryPointQueryResult qa{}, qb{};
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &a, 12000, cudaEnableDefault,
+                                             &qa) == cudaSuccess &&
+            qa == cudaDriverEntryPointSuccess &&
+            cudaGetDriverEntryPointByVersion("cuCtxGetId", &b, 12000, cudaEnableDefault, &qb) ==
+                cudaSuccess &&
+            qb == cudaDriverEntryPointSuccess) {
+            get_current = reinterpret_cast<CtxGetCurrentFn>(a);
+            get_id = reinterpret_cast<CtxGetIdFn>(b);
+        }
+    });
+    if (!get_current || !get_id)
+        return 0;
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS)
+        return 0;
+    return id;
+}
+
+// Device address of g_noalloc_scratch in the current device's context.  It is
+// looked up (cudaGetSymbolAddress, with that device current) on the first
+// call in a context and cached with the context's id; a call from another
+// context of the same device -- after cudaDeviceReset, or under a context the
+// caller made current -- looks it up again, so a cached address is never used
+// in a context it does not belong to.
 int noalloc_scratch(void **ptr)
 {
+    struct Entry {
+        unsigned long long ctx;
+        void *ptr;
+    };
     static std::mutex mu;
-    static void *cache[64] = {nullptr};
+    static Entry cache[64] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64)
         return CADKV_ERR_CUDA;
     std::lock_guard<std::mutex> lock(mu);
-    if (!cache[dev]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p)
-            return CADKV_ERR_CUDA;
-        cache[dev] = p;
+    unsigned long long ctx = current_context_id();
+    if (ctx != 0 && cache[dev].ctx == ctx && cache[dev].ptr) {
+        *ptr = cache[dev].ptr;
+        return CADKV_OK;
     }
-    *ptr = cache[dev];
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p)
+        return CADKV_ERR_CUDA;
+    if (ctx == 0)  // the lookup above made the device's primary context current
+        ctx = current_context_id();
+    cache[dev].ctx = ctx;
+    cache[dev].ptr = ctx != 0 ? p : nullptr;  // without a context id, never reuse
+    *ptr = p;
     return CADKV_OK;
 }
 

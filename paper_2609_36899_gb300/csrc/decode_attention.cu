@@ -238,7 +238,7 @@ __device__ __forceinline__ int slice_of(long long x, long long W, long long T)
     return (int)(((x + 1) * T + W - 1) / W - 1);
 }
 
-// All 128 consumer threads arrive and wait; bounded, abort-aware.
+// All consumer threads (8 warps, 256 threads) arrive and wait; bounded, abort-aware.
 __device__ __forceinline__ bool consumer_sync(uint64_t *bar, uint32_t &phase, volatile int *abort)
 {
     mbar_arrive(bar);

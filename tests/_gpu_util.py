@@ -2,7 +2,10 @@
 the oracle on the same bf16 bits, and compare within the stated tolerances.
 
 Tolerances (decode attention): max |out_gpu - out_oracle| <= 1e-2 and
-|lse_gpu - lse_oracle| <= 1e-3 * |lse_oracle|.  Prefix staging: bit-exact.
+|lse_gpu - lse_oracle| <= 1e-3 * max(|lse_oracle|, 1): relative, with a floor
+of 1 where the reference lse itself comes near zero (a trajectory of one or a
+few tokens whose scores are near zero; there the relative error of even a
+correctly rounded result is unbounded).  Prefix staging: bit-exact.
 """
 import numpy as np
 import torch
@@ -52,7 +55,7 @@ def assert_close(out_gpu, lse_gpu, out_ref, lse_ref, what=""):
         assert np.array_equal(np.isneginf(l), inf_ref), f"{what}: -inf lse mismatch"
         fin = ~inf_ref
         if fin.any():
-            rel = np.abs(l[fin] - lse_ref[fin]) / np.maximum(np.abs(lse_ref[fin]), 1e-30)
+            rel = np.abs(l[fin] - lse_ref[fin]) / np.maximum(np.abs(lse_ref[fin]), 1.0)
             assert rel.max() <= LSE_RTOL, f"{what}: max lse rel err = {rel.max():.3e}"
     return err
 
@@ -108,3 +111,31 @@ def sampled_oracle(batch_dev: DecodeBatch, sample_b):
         pos += p
     q = bf16_bits(batch_dev.q[torch.as_tensor(np.asarray(sample_b), device=batch_dev.q.device)])
     return oracle.decode_attention(q, k, v, table, lens)
+
+
+def full_oracle(batch_dev: DecodeBatch, max_group_bytes=2 << 30):
+    """Oracle for EVERY trajectory of a device-resident batch.
+
+    Trajectories are taken in order, in groups whose K and V pages fit in
+    ``max_group_bytes`` of host memory; each group goes through
+    ``sampled_oracle``.  Returns (out float64 [B, Hq, D], lse float64 [B, Hq]).
+    """
+    lens = batch_dev.context_lens
+    _, hkv, page, d = batch_dev.k_pages.shape
+    page_bytes = 2 * hkv * page * d * 2
+    pages = -(-lens.astype(np.int64) // 16)
+    outs, lses, group, acc = [], [], [], 0
+    for b in range(len(lens)):
+        need = int(pages[b]) * page_bytes
+        if group and acc + need > max_group_bytes:
+            o, l = sampled_oracle(batch_dev, group)
+            outs.append(o)
+            lses.append(l)
+            group, acc = [], 0
+        group.append(b)
+        acc += need
+    if group:
+        o, l = sampled_oracle(batch_dev, group)
+        outs.append(o)
+        lses.append(l)
+    return np.concatenate(outs), np.concatenate(lses)

@@ -9,7 +9,7 @@ import oracle
 import paper_2609_36899_gb300 as cadkv
 from paper_2609_36899_gb300 import STATUS
 from paper_2609_36899_gb300.workloads import MIXED, bf16_bits, make_decode_batch
-from _gpu_util import assert_close, make_batch, sampled_oracle
+from _gpu_util import assert_close, full_oracle, make_batch
 
 pytestmark = pytest.mark.gpu
 
@@ -50,27 +50,45 @@ def test_append_then_attend(g, d):
     assert_close(out, lse, ref, ref_lse, f"append G={g} D={d}")
 
 
-def test_append_full_size_mixed_sampled():
+def test_append_full_size_mixed_every_row():
+    """The whole decode step of the full-size mixed batch (512 trajectories,
+    dynamic-slice path).  The pool after the append equals the oracle's
+    kv_append of the original pool (every trajectory's last page compared bit
+    for bit with the oracle applied to a host copy of it; every other page
+    unchanged), and every output row is within tolerance of the oracle's
+    attention over that pool."""
     batch = make_decode_batch(MIXED, device="cuda")
-    k_new = torch.randn((MIXED.batch, 8, 128), device="cuda").to(torch.bfloat16)
-    v_new = torch.randn((MIXED.batch, 8, 128), device="cuda").to(torch.bfloat16)
+    g = torch.Generator(device="cuda").manual_seed(4242)
+    k_new = torch.randn((MIXED.batch, 8, 128), generator=g, device="cuda").to(torch.bfloat16)
+    v_new = torch.randn((MIXED.batch, 8, 128), generator=g, device="cuda").to(torch.bfloat16)
+    lens = batch.context_lens
+    last = np.array([batch.block_table[b, (int(n) - 1) // 16] for b, n in enumerate(lens)],
+                    dtype=np.int64)
+    assert len(set(last.tolist())) == len(last)      # one distinct page per trajectory
+    last_dev = torch.from_numpy(last).cuda()
+    k_before = batch.k_pages.clone()
+    v_before = batch.v_pages.clone()
     bt = torch.from_numpy(batch.block_table).cuda()
-    cl = torch.from_numpy(batch.context_lens).cuda()
+    cl = torch.from_numpy(lens).cuda()
     out, lse = cadkv.decode_attention_append(batch.q, k_new, v_new, batch.k_pages,
                                              batch.v_pages, bt, cl)
     torch.cuda.synchronize()
-    lens = batch.context_lens
-    sample = sorted({int(np.argmax(lens)), int(np.argmin(lens)), 100, 300})
-    for b in sample:   # the new rows landed in the pool
-        t = int(lens[b]) - 1
-        ph = int(batch.block_table[b, t // 16])
-        assert torch.equal(batch.k_pages[ph, :, t % 16].view(torch.int16),
-                           k_new[b].view(torch.int16))
-        assert torch.equal(batch.v_pages[ph, :, t % 16].view(torch.int16),
-                           v_new[b].view(torch.int16))
-    ref, ref_lse = sampled_oracle(batch, sample)     # reads the updated pool
-    idx = torch.tensor(sample, device="cuda")
-    assert_close(out[idx], lse[idx], ref, ref_lse, "mixed + append")
+    # oracle append on host copies of the last pages, renumbered 0..B-1 (every
+    # page of row b names copy b; only the last one is written)
+    table = np.full_like(batch.block_table, -1)
+    for b, n in enumerate(lens):
+        table[b, :-(-int(n) // 16)] = b
+    kp = bf16_bits(k_before.index_select(0, last_dev)).copy()
+    vp = bf16_bits(v_before.index_select(0, last_dev)).copy()
+    oracle.kv_append(kp, vp, bf16_bits(k_new), bf16_bits(v_new), table, lens)
+    np.testing.assert_array_equal(bf16_bits(batch.k_pages.index_select(0, last_dev)), kp)
+    np.testing.assert_array_equal(bf16_bits(batch.v_pages.index_select(0, last_dev)), vp)
+    for after, before in ((batch.k_pages, k_before), (batch.v_pages, v_before)):
+        changed = (after.view(torch.int16) != before.view(torch.int16)).flatten(1).any(1)
+        assert set(changed.nonzero().flatten().tolist()) <= set(last.tolist())
+    del k_before, v_before
+    ref, ref_lse = full_oracle(batch)               # over the verified pool
+    assert_close(out, lse, ref, ref_lse, "mixed + append, all rows")
     del batch
     torch.cuda.empty_cache()
 

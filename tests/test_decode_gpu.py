@@ -2,8 +2,8 @@
 fp64 oracle, on the same bf16 inputs.
 
 Sizes: the tiny workload in full; the paced / long-tail / mixed workloads at
-reduced batch sizes with their length distributions (full oracle), and at
-their full sizes in the bench's launch configuration on sampled trajectories;
+reduced batch sizes with their length distributions, and at their full sizes
+in the bench's launch configuration, every output row against the oracle;
 plus ragged, empty, maximal and degenerate cases and the method's invariances.
 """
 import numpy as np
@@ -14,8 +14,8 @@ import paper_2609_36899_gb300 as cadkv
 from paper_2609_36899_gb300 import STATUS
 from paper_2609_36899_gb300.workloads import (LONG_TAIL, MIXED, PACED, TINY, DecodeBatch,
                                               bf16_bits, make_decode_batch)
-from _gpu_util import (assert_close, device_tensors, gpu_decode, make_batch,
-                       oracle_decode, sampled_oracle)
+from _gpu_util import (assert_close, device_tensors, full_oracle, gpu_decode, make_batch,
+                       oracle_decode)
 
 pytestmark = pytest.mark.gpu
 
@@ -43,23 +43,35 @@ def test_reduced_workloads_full_oracle(w, bsz):
 
 
 @pytest.mark.parametrize("w", [PACED, LONG_TAIL, MIXED], ids=["paced", "long_tail", "mixed"])
-def test_full_size_sampled(w):
-    """Full-size batch generated on the GPU, every output row finite, and the
-    longest, the shortest and four random trajectories against the oracle."""
+def test_full_size_every_row(w):
+    """Full-size batch generated on the GPU, run in the bench's launch
+    configuration (automatic slicing: the mixed batch takes the dynamic-slice
+    path with multi-CTA merges of its long tails), and EVERY (trajectory,
+    query head) row of out and lse compared with the fp64 oracle."""
     batch = make_decode_batch(w, device="cuda")
     tensors = (batch.q, batch.k_pages, batch.v_pages,
                torch.from_numpy(batch.block_table).cuda(),
                torch.from_numpy(batch.context_lens).cuda())
     out, lse = gpu_decode(batch, tensors=tensors)
-    assert torch.isfinite(out.float()).all()
-    assert torch.isfinite(lse).all()
-    lens = batch.context_lens
-    rng = np.random.Generator(np.random.PCG64(7))
-    sample = sorted(set([int(np.argmax(lens)), int(np.argmin(lens))]
-                        + [int(x) for x in rng.choice(len(lens), 4, replace=False)]))
-    ref, ref_lse = sampled_oracle(batch, sample)
-    idx = torch.tensor(sample, device="cuda")
-    assert_close(out[idx], lse[idx], ref, ref_lse, f"{w.name} sampled {sample}")
+    ref, ref_lse = full_oracle(batch)
+    assert ref.shape == tuple(out.shape)
+    assert_close(out, lse, ref, ref_lse, f"{w.name}, all {len(batch.context_lens)} trajectories")
+    del batch, tensors
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("slice_pages", [61, 4096, 1 << 20])
+def test_mixed_full_size_forced_slices_every_row(slice_pages):
+    """The full-size mixed batch with the work slices forced short (many
+    partials per trajectory-head), at the planner's dynamic-slice length and
+    unsplit: every row against the oracle."""
+    batch = make_decode_batch(MIXED, device="cuda")
+    tensors = (batch.q, batch.k_pages, batch.v_pages,
+               torch.from_numpy(batch.block_table).cuda(),
+               torch.from_numpy(batch.context_lens).cuda())
+    out, lse = gpu_decode(batch, slice_pages=slice_pages, tensors=tensors)
+    ref, ref_lse = full_oracle(batch)
+    assert_close(out, lse, ref, ref_lse, f"mixed, slice_pages={slice_pages}")
     del batch, tensors
     torch.cuda.empty_cache()
 
@@ -235,8 +247,9 @@ def test_workspace_too_small_is_rejected():
 
 
 @pytest.mark.parametrize("b,c", [(32, 16384), (8, 65536), (512, 1024)])
-def test_landscape_cells_sampled(b, c):
-    """Cells of the (B, mean context) landscape sweep, full size, sampled rows."""
+def test_landscape_cells_every_row(b, c):
+    """Cells of the (B, mean context) landscape sweep at full size, every row
+    against the oracle."""
     from paper_2609_36899_gb300.workloads import landscape_workload
     w = landscape_workload(b, c)
     batch = make_decode_batch(w, device="cuda")
@@ -244,18 +257,17 @@ def test_landscape_cells_sampled(b, c):
                torch.from_numpy(batch.block_table).cuda(),
                torch.from_numpy(batch.context_lens).cuda())
     out, lse = gpu_decode(batch, tensors=tensors)
-    lens = batch.context_lens
-    sample = sorted({int(np.argmax(lens)), int(np.argmin(lens)), len(lens) // 2})
-    ref, ref_lse = sampled_oracle(batch, sample)
-    idx = torch.tensor(sample, device="cuda")
-    assert_close(out[idx], lse[idx], ref, ref_lse, w.name)
+    ref, ref_lse = full_oracle(batch)
+    assert_close(out, lse, ref, ref_lse, w.name)
+    del batch, tensors
+    torch.cuda.empty_cache()
 
 
 @pytest.mark.parametrize("comp", ["equal", "lognormal", "bimodal", "one_giant"])
-def test_composition_cells_sampled(comp):
+def test_composition_cells_every_row(comp):
     """The within-batch composition sweep at B = 128, mean 4096 (full size as
-    benched): the longest trajectory (half of all tokens for one_giant), the
-    shortest and one in the middle against the oracle."""
+    benched; one_giant gives one trajectory half of all tokens), every row
+    against the oracle."""
     from paper_2609_36899_gb300.workloads import composition_workload
     w = composition_workload(128, 4096, comp)
     batch = make_decode_batch(w, device="cuda")
@@ -263,12 +275,8 @@ def test_composition_cells_sampled(comp):
                torch.from_numpy(batch.block_table).cuda(),
                torch.from_numpy(batch.context_lens).cuda())
     out, lse = gpu_decode(batch, tensors=tensors)
-    assert torch.isfinite(out.float()).all() and torch.isfinite(lse).all()
-    lens = batch.context_lens
-    sample = sorted({int(np.argmax(lens)), int(np.argmin(lens)), len(lens) // 2})
-    ref, ref_lse = sampled_oracle(batch, sample)
-    idx = torch.tensor(sample, device="cuda")
-    assert_close(out[idx], lse[idx], ref, ref_lse, w.name)
+    ref, ref_lse = full_oracle(batch)
+    assert_close(out, lse, ref, ref_lse, w.name)
     del batch, tensors
     torch.cuda.empty_cache()
 

@@ -4,10 +4,12 @@ nearly all HBM for its KV cache up front, or a plugin with no access to its
 host framework's allocator).  It uses the library's built-in scratch array
 instead of a caller workspace.
 
-Called here through the C ABI (ctypes, no binding wrapper) and compared with
-decode_attention (caller workspace) on the same inputs, within the tolerances
-of the other parity tests, on two calls in a row.  This file is collected last
-so that a failure here never hides another test's result.
+Called here through the C ABI (ctypes, no binding wrapper) and compared,
+within the tolerances of the other parity tests, with the fp64 oracle and with
+decode_attention (caller workspace) on the same inputs, on two calls in a row,
+and after other problems that left their contents in the shared scratch.  This
+file is collected last so that a failure here never hides another test's
+result.
 """
 import ctypes
 
@@ -15,13 +17,15 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 import paper_2609_36899_gb300 as cadkv
 from paper_2609_36899_gb300 import STATUS
+from paper_2609_36899_gb300.workloads import bf16_bits
 
 pytestmark = pytest.mark.gpu
 
 OUT_ATOL = 1e-2
-LSE_RTOL = 1e-3
+LSE_RTOL = 1e-3   # relative to max(|lse|, 1), as in the other parity tests
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -66,8 +70,25 @@ def _compare(out, lse, ref_out, ref_lse):
     assert err <= OUT_ATOL, err
     fin = torch.isfinite(ref_lse)
     assert torch.equal(torch.isneginf(lse), torch.isneginf(ref_lse))
-    rel = ((lse[fin] - ref_lse[fin]).abs() / ref_lse[fin].abs()).max().item()
+    rel = ((lse[fin] - ref_lse[fin]).abs() / ref_lse[fin].abs().clamp(min=1.0)).max().item()
     assert rel <= LSE_RTOL, rel
+
+
+def _compare_oracle(out, lse, q, k, v, bt, cl):
+    """Against the fp64 oracle on the same bf16 bits."""
+    ref, ref_lse = oracle.decode_attention(bf16_bits(q), bf16_bits(k), bf16_bits(v),
+                                           bt.cpu().numpy(), cl.cpu().numpy())
+    o = out.float().cpu().numpy().astype(np.float64)
+    assert np.all(np.isfinite(o))
+    err = np.abs(o - ref).max(initial=0.0)
+    assert err <= OUT_ATOL, err
+    l = lse.cpu().numpy().astype(np.float64)
+    inf_ref = np.isneginf(ref_lse)
+    assert np.array_equal(np.isneginf(l), inf_ref)
+    fin = ~inf_ref
+    if fin.any():
+        rel = (np.abs(l[fin] - ref_lse[fin]) / np.maximum(np.abs(ref_lse[fin]), 1.0)).max()
+        assert rel <= LSE_RTOL, rel
 
 
 @pytest.mark.parametrize("lens,hq,hkv,d", [
@@ -83,6 +104,7 @@ def test_noalloc_matches_workspace_entry_point_twice(lens, hq, hkv, d):
         assert _call_noalloc(q, k, v, bt, cl, out, lse) == 0
         torch.cuda.synchronize()
         _compare(out, lse, ref_out, ref_lse)
+        _compare_oracle(out, lse, q, k, v, bt, cl)
 
 
 def test_noalloc_after_a_different_problem():
@@ -96,6 +118,24 @@ def test_noalloc_after_a_different_problem():
         assert _call_noalloc(q, k, v, bt, cl, out, lse) == 0
         torch.cuda.synchronize()
         _compare(out, lse, ref_out, ref_lse)
+        _compare_oracle(out, lse, q, k, v, bt, cl)
+
+
+def test_noalloc_many_partials_after_a_bigger_problem():
+    """A long trajectory next to short ones is cut into many slices, so its
+    (trajectory, KV head) units go through several partial slots and arrival
+    counters of the shared scratch; it runs right after a bigger problem left
+    its own partials and counters there, and twice in a row, each time against
+    the oracle."""
+    big = _inputs([40000, 9000, 300, 77, 20000, 5, 60000, 1200], 64, 8, 128, seed=11)
+    small = _inputs([60000, 20, 33, 100, 1], 32, 8, 128, seed=12)
+    for q, k, v, bt, cl in (big, small, small):
+        out = torch.full_like(q, float("nan"))
+        lse = torch.full((q.shape[0], q.shape[1]), float("nan"), dtype=torch.float32,
+                         device="cuda")
+        assert _call_noalloc(q, k, v, bt, cl, out, lse) == 0
+        torch.cuda.synchronize()
+        _compare_oracle(out, lse, q, k, v, bt, cl)
 
 
 def test_noalloc_rejects_problems_beyond_the_scratch():
