@@ -49,7 +49,7 @@ METRIC = "decode-attention achieved HBM GB/s (% of 8 TB/s) and decode steps/s pe
 NOMINAL_HBM_GBS = 8000.0
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
-PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "decode_attention_kernel_paced_b256.md")
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "decode_attention_kernel_mixed_b512_dram.md")
 STAGE_PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "stage_copy_kernel_staging_8traj_1layer.md")
 KERNEL_SOURCE = os.path.join(ROOT, "paper_2609_36899_gb300", "csrc", "decode_attention.cu")
 STAGE_SOURCE = os.path.join(ROOT, "paper_2609_36899_gb300", "csrc", "prefix_stage.cu")
@@ -623,34 +623,97 @@ def read_probe(buf, reps=10):
     return buf.numel() * buf.element_size() * reps / (e0.elapsed_time(e1) * 1e-3) / 1e9
 
 
+L2_BYTES = 129 << 20   # GB300 L2 (per GPU)
+
+
 def _decode_cell(w, device, steps, warmup):
     """Back-to-back decode steps of one workload: GB/s, time and steps/s, from
-    the better of two timed runs of ``steps`` steps (both are reported)."""
+    the better of two timed runs of ``steps`` steps (both are reported).
+
+    A decode step is one layer's attention.  As in a model's layer loop, step i
+    reads layer i mod L of L layers of KV pages (same lengths and tables, other
+    values), with L chosen so that the L layers together exceed three times the
+    L2, so that no step finds its pages in L2 (L = 1 when one layer already
+    does).  ``same_layer`` repeats layer 0 instead, the way the cell was timed
+    before; small cells then stream from L2.
+
+    Eager: one decode_attention call per step from Python, so a step can be no
+    shorter than the host's time to issue it (host_us_per_call).  Graph: the
+    same calls captured once in a CUDA graph and replayed, as a serving engine
+    issues its decode steps: the device time."""
     batch = make_decode_batch(w, device=device)
     tensors = _tensors(batch, device)
-    stream = torch.cuda.current_stream(device)
+    stream = torch.cuda.Stream(device)
     q, k, v, bt, cl, out, lse, ws = tensors
-    for _ in range(warmup):
-        cadkv.decode_attention(q, k, v, bt, cl, out=out, lse=lse, workspace=ws, stream=stream)
-    runs = []
-    for _ in range(2):   # a cell timed right after much larger ones was sometimes slow once
+    layer_bytes = 2 * k.numel() * k.element_size()
+    n_layers = max(1, min(32, -(-3 * L2_BYTES // layer_bytes)))
+    layers = [(k, v)]
+    for l in range(1, n_layers):
+        g = torch.Generator(device=device).manual_seed(w.seed * 1000 + l)
+        layers.append(tuple(torch.randn(k.shape, generator=g, device=device,
+                                        dtype=torch.float32).to(torch.bfloat16)
+                            for _ in range(2)))
+
+    def step(l):
+        kl, vl = layers[l]
+        cadkv.decode_attention(q, kl, vl, bt, cl, out=out, lse=lse, workspace=ws, stream=stream)
+
+    def timed(fn, reps):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        for _ in range(steps):   # back to back: the planner/attention overlap is kept
-            cadkv.decode_attention(q, k, v, bt, cl, out=out, lse=lse, workspace=ws, stream=stream)
+        fn()
         e1.record(stream)
         torch.cuda.synchronize()
-        runs.append(e0.elapsed_time(e1) / steps)
-    step_ms = min(runs)
+        return e0.elapsed_time(e1) / reps
+
+    def rotating():
+        for i in range(steps):   # back to back: the planner/attention overlap is kept
+            step(i % n_layers)
+
+    def same_layer():
+        for _ in range(steps):
+            step(0)
+
+    res = {}
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for _ in range(warmup):
+            step(0)
+        torch.cuda.synchronize()
+        for name, loop in (("rotating", rotating), ("same_layer", same_layer)):
+            # a cell timed right after much larger ones was sometimes slow once
+            runs = [timed(loop, steps) for _ in range(2)]
+            t0 = time.perf_counter()
+            loop()
+            host_us = (time.perf_counter() - t0) / steps * 1e6
+            torch.cuda.synchronize()
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=stream):
+                loop()
+            graph.replay()
+            torch.cuda.synchronize()
+            graph_runs = [timed(graph.replay, steps) for _ in range(2)]
+            del graph
+            res[name] = (runs, graph_runs, host_us)
     nbytes = decode_bytes(batch.context_lens, w.num_q_heads, w.num_kv_heads, w.head_dim)
-    cell = {"gbps": round(nbytes / (step_ms * 1e-3) / 1e9, 1),
-            "ms_per_step": round(step_ms, 4),
-            "ms_per_step_runs": [round(r, 4) for r in runs],
-            "steps_per_s": round(1e3 / step_ms, 1),
-            "tokens_per_s_per_layer": round(w.batch * 1e3 / step_ms, 1),
-            "max_context": int(batch.context_lens.max()),
-            "status": cadkv.decode_attention_status(ws)}
-    del batch, tensors
+
+    def summary(runs, graph_runs, host_us):
+        ms, gms = min(runs), min(graph_runs)
+        return {"gbps": round(nbytes / (ms * 1e-3) / 1e9, 1), "ms_per_step": round(ms, 4),
+                "ms_per_step_runs": [round(r, 4) for r in runs],
+                "steps_per_s": round(1e3 / ms, 1),
+                "host_us_per_call": round(host_us, 2),
+                "graph": {"gbps": round(nbytes / (gms * 1e-3) / 1e9, 1),
+                          "ms_per_step": round(gms, 4),
+                          "ms_per_step_runs": [round(r, 4) for r in graph_runs]}}
+
+    cell = summary(*res["rotating"])
+    cell["tokens_per_s_per_layer"] = round(w.batch * 1e3 / cell["ms_per_step"], 1)
+    cell["layers_rotated"] = n_layers
+    cell["same_layer"] = summary(*res["same_layer"])
+    cell["max_context"] = int(batch.context_lens.max())
+    cell["status"] = cadkv.decode_attention_status(ws, stream)
+    del layers, batch, tensors, q, k, v, bt, cl, out, lse, ws
     torch.cuda.empty_cache()
     return cell
 

@@ -110,13 +110,14 @@ def _check(func: str, rc: int):
 
 
 def _ptr(t):
-    return None if t is None else ctypes.c_void_p(t.data_ptr())
+    # a plain int: the c_void_p argtypes convert it (cheaper than a c_void_p object)
+    return None if t is None else t.data_ptr()
 
 
 def _stream(stream, device):
     if stream is None:
         stream = torch.cuda.current_stream(device)
-    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
 
 
 def _need(t: torch.Tensor, name: str, dtype, ndim: int | None = None, device=None):
@@ -170,8 +171,8 @@ def _outputs(q, out, lse, want_lse, workspace, batch, hq, hkv, d, max_pages):
         lse = torch.empty((batch, hq), dtype=torch.float32, device=q.device)
     elif lse is not None:
         _need(lse, "lse", torch.float32, 2, q.device)
-    need = decode_attention_workspace_size(batch, hq, hkv, d, max_pages)
     if workspace is None:
+        need = decode_attention_workspace_size(batch, hq, hkv, d, max_pages)
         workspace = torch.empty(max(need, 1), dtype=torch.uint8, device=q.device)
     else:
         _need(workspace, "workspace", torch.uint8, 1, q.device)

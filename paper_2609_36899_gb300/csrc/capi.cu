@@ -24,7 +24,7 @@ struct cadkv_pool {
 
 namespace {
 
-constexpr int kAbiVersion = (1 << 16) | 0;
+constexpr int kAbiVersion = (1 << 16) | 1;
 
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
@@ -112,6 +112,46 @@ int encode_pages_map(CUtensorMap *map, const void *pages, int num_pages, int num
     return r == CUDA_SUCCESS ? CADKV_OK : CADKV_ERR_CUDA;
 }
 
+// encode_pages_map through a small per-thread cache: a serving loop calls
+// decode attention with the same page pools over and over, and encoding a
+// tensor map costs host time on every call.  A map depends only on its inputs
+// (the pool pointer and geometry), so equal inputs give an equal map.
+int encode_pages_map_cached(CUtensorMap *map, const void *pages, int num_pages, int num_kv_heads,
+                            int head_dim, bool allow_whole, int *whole_block)
+{
+    struct Entry {
+        const void *pages;
+        int num_pages, num_kv_heads, head_dim, allow_whole, whole;
+        CUtensorMap map;
+    };
+    constexpr int kEntries = 8;
+    thread_local Entry cache[kEntries] = {};
+    thread_local int next = 0;
+    for (int i = 0; i < kEntries; ++i) {
+        const Entry &e = cache[i];
+        if (e.pages == pages && e.num_pages == num_pages && e.num_kv_heads == num_kv_heads &&
+            e.head_dim == head_dim && e.allow_whole == (int)allow_whole) {
+            *map = e.map;
+            *whole_block = e.whole;
+            return CADKV_OK;
+        }
+    }
+    const int rc = encode_pages_map(map, pages, num_pages, num_kv_heads, head_dim, allow_whole,
+                                    whole_block);
+    if (rc == CADKV_OK) {
+        Entry &e = cache[next];
+        next = (next + 1) % kEntries;
+        e.pages = pages;
+        e.num_pages = num_pages;
+        e.num_kv_heads = num_kv_heads;
+        e.head_dim = head_dim;
+        e.allow_whole = (int)allow_whole;
+        e.whole = *whole_block;
+        e.map = *map;
+    }
+    return rc;
+}
+
 struct DecodeShape {
     int batch, num_q_heads, num_kv_heads, head_dim, page_size, num_pages, max_pages;
 };
@@ -142,6 +182,13 @@ int workspace_carve(const DecodeShape &s, void *workspace, size_t workspace_byte
     if (!workspace || !aligned(workspace, kWorkspaceAlign) || workspace_bytes < L->total)
         return CADKV_ERR_WORKSPACE;
     return CADKV_OK;
+}
+
+// Threads of the planner launch: small batches without a fused append are
+// planned by a CTA small enough to share an SM with an attention CTA.
+int plan_threads(int batch, bool append)
+{
+    return !append && batch <= kSmallPlanMaxBatch ? kPlanThreadsSmall : kPlanThreads;
 }
 
 // New-token rows written into the pool before attention (decode_attention_append).
@@ -188,6 +235,7 @@ int plan_impl(const int32_t *context_lens, void *out, float *lse, const DecodeSh
     p.max_pages = s.max_pages;
     p.slice_cap = L.slice_cap;
     p.slice_pages = slice_pages;
+    p.threads = plan_threads(s.batch, append != nullptr);
     if (append) {
         p.k_new = static_cast<const __nv_bfloat16 *>(append->k_new);
         p.v_new = static_cast<const __nv_bfloat16 *>(append->v_new);
@@ -236,16 +284,16 @@ int run_impl(const void *q, const void *k_pages, const void *v_pages,
         return rc;
     CUtensorMap kmap, vmap;
     int k_whole = 0, v_whole = 0;
-    if (encode_pages_map(&kmap, k_pages, s.num_pages, s.num_kv_heads, s.head_dim, true,
-                         &k_whole) != CADKV_OK ||
-        encode_pages_map(&vmap, v_pages, s.num_pages, s.num_kv_heads, s.head_dim, true,
-                         &v_whole) != CADKV_OK)
+    if (encode_pages_map_cached(&kmap, k_pages, s.num_pages, s.num_kv_heads, s.head_dim, true,
+                                &k_whole) != CADKV_OK ||
+        encode_pages_map_cached(&vmap, v_pages, s.num_pages, s.num_kv_heads, s.head_dim, true,
+                                &v_whole) != CADKV_OK)
         return CADKV_ERR_CUDA;
     if (k_whole != v_whole) {  // both maps must use the same box shape
-        if (encode_pages_map(&kmap, k_pages, s.num_pages, s.num_kv_heads, s.head_dim, false,
-                             &k_whole) != CADKV_OK ||
-            encode_pages_map(&vmap, v_pages, s.num_pages, s.num_kv_heads, s.head_dim, false,
-                             &v_whole) != CADKV_OK)
+        if (encode_pages_map_cached(&kmap, k_pages, s.num_pages, s.num_kv_heads, s.head_dim,
+                                    false, &k_whole) != CADKV_OK ||
+            encode_pages_map_cached(&vmap, v_pages, s.num_pages, s.num_kv_heads, s.head_dim,
+                                    false, &v_whole) != CADKV_OK)
             return CADKV_ERR_CUDA;
     }
     uint8_t *ws = static_cast<uint8_t *>(workspace);

@@ -80,16 +80,20 @@ __device__ __forceinline__ void append_rows(const PlanParams &p)
         dst[c] = src[c];
 }
 
-__global__ void __launch_bounds__(1024, 1) plan_kernel(const PlanParams p)
+__global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(const PlanParams p)
 {
-    // Let the attention kernel launch now: it sets up its shared memory and then
-    // waits (griddepcontrol.wait) for this whole grid to finish before it reads
-    // anything the planner or the append CTAs write.
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    // This grid is itself launched programmatically, so it may start while the
-    // previous kernel on the stream (often the last decode step) is finishing:
-    // nothing is read or written here before that kernel's writes are visible.
+    // This grid is launched programmatically, so it may start while the previous
+    // kernel on the stream (often the last decode step's attention kernel, which
+    // lets it launch as soon as it starts) is still running: nothing is read or
+    // written here before that kernel's writes are visible.
     asm volatile("griddepcontrol.wait;" ::: "memory");
+    // Now let the attention kernel launch: it sets up its shared memory and then
+    // waits (griddepcontrol.wait) for this whole grid to finish before it reads
+    // anything the planner or the append CTAs write.  Triggered before the wait
+    // above, its CTAs took the SMs of the previous step's CTAs as they left and
+    // the small-batch steps ran slower (29.5 against 27.3 us for 32 x 1,024
+    // tokens in a CUDA graph).
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (blockIdx.x > 0) {
         append_rows(p);
         return;
@@ -97,6 +101,7 @@ __global__ void __launch_bounds__(1024, 1) plan_kernel(const PlanParams p)
     __shared__ long long warp_sums[32];
     __shared__ long long carry_s;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int nthreads = blockDim.x, nwarps = nthreads >> 5;
     const int max_len = p.max_pages * kPageSize;
     if (tid == 0) {
         p.hdr->status = 0;
@@ -104,7 +109,7 @@ __global__ void __launch_bounds__(1024, 1) plan_kernel(const PlanParams p)
     }
     __syncthreads();
 
-    for (int base = 0; base < p.batch; base += 1024) {
+    for (int base = 0; base < p.batch; base += nthreads) {
         const int b = base + tid;
         long long pages = 0;
         if (b < p.batch) {
@@ -136,7 +141,7 @@ __global__ void __launch_bounds__(1024, 1) plan_kernel(const PlanParams p)
             warp_sums[warp] = v;
         __syncthreads();
         if (warp == 0) {
-            long long w = warp_sums[lane];
+            long long w = lane < nwarps ? warp_sums[lane] : 0;
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {
                 long long u = __shfl_up_sync(kFull, w, o);
@@ -151,30 +156,22 @@ __global__ void __launch_bounds__(1024, 1) plan_kernel(const PlanParams p)
         if (b < p.batch)
             p.page_prefix[b] = incl - pages;
         __syncthreads();
-        if (tid == 1023)
+        if (tid == nthreads - 1)
             carry_s = incl;
         __syncthreads();
     }
-    for (int i = tid; i < p.batch * p.num_kv_heads; i += 1024)
+    for (int i = tid; i < p.batch * p.num_kv_heads; i += nthreads)
         p.unit_counter[i] = 0;
     if (tid == 0) {
         const long long total = carry_s;
         p.page_prefix[p.batch] = total;
         const long long W = total * p.num_kv_heads;
-        const long long unit = p.slice_pages > 0 ? p.slice_pages : kMinSlicePages;
-        long long T = (W + unit - 1) / unit;
         // Dynamic slices (several per CTA) absorb per-SM speed differences, but
         // each costs a start-up chain of dependent loads (slice, trajectory,
         // table) and a pipeline fill; below ~4K page-heads per CTA that cost wins,
         // so automatic slicing gives each CTA one equal slice there.
-        const long long ctas = p.slice_cap / kSlicesPerCta;
-        const long long cap = (p.slice_pages > 0 || W > kOneSliceMaxPerCta * ctas) ? p.slice_cap : ctas;
-        if (T > cap)
-            T = cap;
-        if (T < 1)
-            T = 1;
         p.hdr->total_work = W;
-        p.hdr->num_slices = (int)T;
+        p.hdr->num_slices = (int)plan_num_slices(W, p.slice_pages, p.slice_cap);
         p.hdr->slice_counter = 0;
     }
 }
@@ -255,6 +252,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     using C = AttnConfig<D>;
     constexpr int S = C::kStages;
     static_assert(kIssueGroup <= S, "a parallel issue group must not reuse a stage");
+    // The next decode step's planner may launch now: it waits (griddepcontrol.wait)
+    // for this whole grid before it touches memory, so its launch latency hides
+    // behind this step instead of following it.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     // Page i of a segment goes to consumer warp i % kNumConsumerWarps and lands in
     // stage (k + i) % S.  With S a multiple of the warp count, the next use of a
     // stage within a segment belongs to the warp that released its last use, so
@@ -818,7 +819,7 @@ cudaError_t launch_plan(const PlanParams &p, cudaStream_t stream)
     // tail; it waits for that kernel's writes before touching memory.
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(1 + append_ctas);
-    cfg.blockDim = dim3(1024);
+    cfg.blockDim = dim3(p.threads > 0 ? p.threads : kPlanThreads);
     cfg.dynamicSmemBytes = 0;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];

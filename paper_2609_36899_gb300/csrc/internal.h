@@ -43,6 +43,28 @@ constexpr int kMinSlicePages = 16; // auto slicing never cuts finer than this
 constexpr long long kOneSliceMaxPerCta = 4096;  // page-heads per CTA up to which auto
                                                 // slicing gives each CTA a single slice
 constexpr size_t kWorkspaceAlign = 256;
+// Batches up to this size are planned by a 256-thread CTA (kPlanThreadsSmall)
+// instead of 1024: it fits on an SM beside an attention CTA, so the planner of
+// the next decode step can launch while this step's attention kernel still
+// runs and wait there, and no attention CTA waits for an SM behind it.
+constexpr int kSmallPlanMaxBatch = 2048;
+
+// Work slices T of W flattened page-heads: one equal slice per CTA while a CTA
+// would hold at most kOneSliceMaxPerCta page-heads, up to kSlicesPerCta per CTA
+// above that, or ceil(W / slice_pages) when forced, never more than slice_cap
+// and never fewer than one.
+__host__ __device__ inline long long plan_num_slices(long long W, int slice_pages, int slice_cap)
+{
+    const long long unit = slice_pages > 0 ? slice_pages : kMinSlicePages;
+    long long T = (W + unit - 1) / unit;
+    const long long ctas = slice_cap / kSlicesPerCta;
+    const long long cap = (slice_pages > 0 || W > kOneSliceMaxPerCta * ctas) ? slice_cap : ctas;
+    if (T > cap)
+        T = cap;
+    if (T < 1)
+        T = 1;
+    return T;
+}
 
 // Header at the start of a decode-attention or staging workspace.
 struct alignas(64) WorkspaceHeader {
@@ -87,9 +109,13 @@ struct PlanParams {
     __nv_bfloat16 *k_pages, *v_pages;
     const int *block_table;
     int num_pages;
+    int threads;        // threads per CTA: kPlanThreadsSmall for small batches without a
+                        // fused append (the append CTAs need kPlanThreads)
 };
 
 constexpr int kAppendRowsPerCta = 32;  // one warp per (trajectory, KV head)
+constexpr int kPlanThreads = 1024;
+constexpr int kPlanThreadsSmall = 256;
 
 struct AttnParams {
     const __nv_bfloat16 *q;
