@@ -624,6 +624,7 @@ def read_probe(buf, reps=10):
 
 
 L2_BYTES = 129 << 20   # GB300 L2 (per GPU)
+LAYERS_PER_ITERATION = 36  # Qwen3-8B, the paper's main rollout model
 
 
 def _decode_cell(w, device, steps, warmup):
@@ -635,12 +636,15 @@ def _decode_cell(w, device, steps, warmup):
     values), with L chosen so that the L layers together exceed three times the
     L2, so that no step finds its pages in L2 (L = 1 when one layer already
     does).  ``same_layer`` repeats layer 0 instead, the way the cell was timed
-    before; small cells then stream from L2.
+    before; small cells then stream from L2.  ``plan_per_iteration`` plans once
+    per LAYERS_PER_ITERATION steps (one decode iteration of a model of that
+    depth: the plan depends only on the lengths) and runs each step on it.
 
-    Eager: one decode_attention call per step from Python, so a step can be no
-    shorter than the host's time to issue it (host_us_per_call).  Graph: the
-    same calls captured once in a CUDA graph and replayed, as a serving engine
-    issues its decode steps: the device time."""
+    Eager: one call per step from Python (a DecodeStep, the binding's prepared
+    form of decode_attention), so a step can be no shorter than the host's time
+    to issue it (host_us_per_call).  Graph: the same calls captured once in a
+    CUDA graph and replayed, as a serving engine issues its decode steps: the
+    device time."""
     batch = make_decode_batch(w, device=device)
     tensors = _tensors(batch, device)
     stream = torch.cuda.Stream(device)
@@ -654,9 +658,15 @@ def _decode_cell(w, device, steps, warmup):
                                         dtype=torch.float32).to(torch.bfloat16)
                             for _ in range(2)))
 
+    # one prepared call per layer: the tensors are checked and marshalled once
+    calls = [cadkv.DecodeStep(q, kl, vl, bt, cl, out, lse, ws, stream=stream)
+             for kl, vl in layers]
+    plan = cadkv.DecodeStep(q, k, v, bt, cl, out, lse, ws, stream=stream, launch="plan")
+    runs_only = [cadkv.DecodeStep(q, kl, vl, bt, cl, out, lse, ws, stream=stream, launch="run")
+                 for kl, vl in layers]
+
     def step(l):
-        kl, vl = layers[l]
-        cadkv.decode_attention(q, kl, vl, bt, cl, out=out, lse=lse, workspace=ws, stream=stream)
+        calls[l]()
 
     def timed(fn, reps):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -674,13 +684,22 @@ def _decode_cell(w, device, steps, warmup):
         for _ in range(steps):
             step(0)
 
+    def planned_per_iteration():
+        # a decode iteration of a model with LAYERS_PER_ITERATION layers plans
+        # once and runs every layer on that plan
+        for i in range(steps):
+            if i % LAYERS_PER_ITERATION == 0:
+                plan()
+            runs_only[i % n_layers]()
+
     res = {}
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
         for _ in range(warmup):
             step(0)
         torch.cuda.synchronize()
-        for name, loop in (("rotating", rotating), ("same_layer", same_layer)):
+        for name, loop in (("rotating", rotating), ("same_layer", same_layer),
+                           ("plan_per_iteration", planned_per_iteration)):
             # a cell timed right after much larger ones was sometimes slow once
             runs = [timed(loop, steps) for _ in range(2)]
             t0 = time.perf_counter()
@@ -711,9 +730,10 @@ def _decode_cell(w, device, steps, warmup):
     cell["tokens_per_s_per_layer"] = round(w.batch * 1e3 / cell["ms_per_step"], 1)
     cell["layers_rotated"] = n_layers
     cell["same_layer"] = summary(*res["same_layer"])
+    cell["plan_per_iteration"] = summary(*res["plan_per_iteration"])
     cell["max_context"] = int(batch.context_lens.max())
     cell["status"] = cadkv.decode_attention_status(ws, stream)
-    del layers, batch, tensors, q, k, v, bt, cl, out, lse, ws
+    del calls, plan, runs_only, layers, batch, tensors, q, k, v, bt, cl, out, lse, ws
     torch.cuda.empty_cache()
     return cell
 

@@ -171,7 +171,18 @@ int decode_attention_split(const void *q, const void *k_pages, const void *v_pag
 /*
  * The two launches of decode_attention, exposed separately so a caller can
  * time or graph-capture them apart.  decode_attention_run must follow
- * decode_attention_plan on the same stream with identical arguments.
+ * decode_attention_plan on the same stream with the same context_lens,
+ * sizes and workspace.
+ *
+ * One plan serves several runs.  The plan depends only on the lengths, so a
+ * decode step of an L-layer model plans once and runs once per layer, each
+ * run with that layer's q, k_pages, v_pages, block_table (same width), out
+ * and lse, one after another on the stream: every run leaves the workspace's
+ * counters as the plan left them, and writes all of its outputs (out = 0 and
+ * lse = -inf for trajectories without pages) itself.  Plan again when the
+ * lengths change, when another problem used the workspace, or after a run
+ * whose status word reports an error.  The status word keeps the first error
+ * of any run since the plan.
  */
 int decode_attention_plan(const int32_t *context_lens, void *out, float *lse,
                           int batch, int num_q_heads, int num_kv_heads,

@@ -11,7 +11,7 @@ for sm_103a, C ABI in ``include/cadkv.h``).  Build it with
 ``python -m paper_2609_36899_gb300.build``.
 """
 from ._binding import (  # noqa: F401
-    STATUS, CadkvError, KVPool, LibraryMissing, cadkv_hbm_read_probe, cadkv_wait_selftest,
+    STATUS, CadkvError, DecodeStep, KVPool, LibraryMissing, cadkv_hbm_read_probe, cadkv_wait_selftest,
     decode_attention,
     decode_attention_append, decode_attention_noalloc, decode_attention_plan, decode_attention_run, decode_attention_status,
     decode_attention_workspace_size, header_functions, kv_prefix_load,

@@ -200,6 +200,51 @@ def decode_attention(q, k_pages, v_pages, block_table, context_lens, out=None, l
     return out, lse
 
 
+class DecodeStep:
+    """decode_attention over fixed buffers, validated and marshalled once.
+
+    A serving loop calls decode attention on the same buffers step after step
+    (the values change, the tensors do not).  This object checks the tensors
+    once, keeps references to them, and each call passes the stored pointers
+    straight to the C entry point, so a step costs the host little more than
+    the library's own launch work.  Calling it after any of the tensors was
+    resized or reallocated is an error the object cannot see: build a new one.
+    """
+
+    def __init__(self, q, k_pages, v_pages, block_table, context_lens, out, lse, workspace,
+                 slice_pages: int = 0, stream=None, launch: str = "both"):
+        """launch: "both" (decode_attention: plan and attention), "plan" or
+        "run" (decode_attention_plan / decode_attention_run alone, e.g. one
+        plan per decode step and one run per layer)."""
+        batch, hq, hkv, d, page, num_pages, max_pages = _decode_args(
+            q, k_pages, v_pages, block_table, context_lens)
+        out, lse, workspace = _outputs(q, out, lse, lse is not None, workspace, batch, hq, hkv,
+                                       d, max_pages)
+        self.tensors = (q, k_pages, v_pages, block_table, context_lens, out, lse, workspace)
+        st = _stream(stream, q.device)
+        lib = library()
+        if launch == "plan":
+            self._name, self._fn = "decode_attention_plan", lib.decode_attention_plan
+            self._args = (_ptr(context_lens), _ptr(out), _ptr(lse), batch, hq, hkv, d,
+                          max_pages, int(slice_pages), _ptr(workspace), workspace.numel(), st)
+            return
+        head = (_ptr(q), _ptr(k_pages), _ptr(v_pages), _ptr(block_table), _ptr(context_lens),
+                _ptr(out), _ptr(lse), batch, hq, hkv, d, page, num_pages, max_pages)
+        if launch == "run":
+            self._name, self._fn = "decode_attention_run", lib.decode_attention_run
+            self._args = head + (_ptr(workspace), workspace.numel(), st)
+        elif launch == "both":
+            self._name, self._fn = "decode_attention", lib.decode_attention_split
+            self._args = head + (int(slice_pages), _ptr(workspace), workspace.numel(), st)
+        else:
+            raise ValueError("launch must be 'both', 'plan' or 'run'")
+
+    def __call__(self):
+        rc = self._fn(*self._args)
+        if rc != 0:
+            raise CadkvError(self._name, rc)
+
+
 def decode_attention_append(q, k_new, v_new, k_pages, v_pages, block_table, context_lens,
                             out=None, lse=None, workspace=None, want_lse: bool = True,
                             stream=None):

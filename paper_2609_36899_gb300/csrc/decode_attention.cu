@@ -173,6 +173,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(const PlanParams 
         p.hdr->total_work = W;
         p.hdr->num_slices = (int)plan_num_slices(W, p.slice_pages, p.slice_cap);
         p.hdr->slice_counter = 0;
+        p.hdr->exit_counter = 0;
     }
 }
 
@@ -330,8 +331,22 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     slice = (int)gridDim.x + atomicAdd(&p.hdr->slice_counter, 1);
                 slice = __shfl_sync(kFull, slice, 0);
             }
-            if (slice >= T)
+            if (slice >= T) {
+                // This CTA fetches no more slices.  The last CTA to get here puts the
+                // slice counter back to zero, so that the next attention launch over
+                // the same plan starts from a clean counter (acq_rel: every other
+                // CTA's fetches happened before its increment).
+                if (lane == 0) {
+                    int old;
+                    asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], 1;"
+                                 : "=r"(old) : "l"(&p.hdr->exit_counter) : "memory");
+                    if (old == (int)gridDim.x - 1) {
+                        p.hdr->slice_counter = 0;
+                        p.hdr->exit_counter = 0;
+                    }
+                }
                 break;
+            }
             const long long s0 = slice_begin(slice, W, T), s1 = slice_begin(slice + 1, W, T);
             if (s0 >= s1)
                 continue;
@@ -484,7 +499,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     // ================================ consumer warps ================================
     const int g = lane >> 2, t = lane & 3;          // mma fragment coordinates
     const int mi = lane >> 3, rr = lane & 7;        // ldmatrix: matrix index, row in matrix
-    const int ct = tid;                             // consumer thread 0..127
+    const int ct = tid;                             // consumer thread 0..255
     uint32_t k = 0, sc = 0, cphase = 0;
     bool ok = true;
     SegDesc pd{};         // the last partial whose unit may still need its merge
@@ -534,11 +549,40 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             *is_last_flag = (pend_old == pd.count - 1) ? 1 : 0;
         if (!consumer_sync(cons_bar, cphase, abort_flag))
             return false;
-        if (*is_last_flag)
+        if (*is_last_flag) {
             merge_unit(pd);
+            // every partial of the unit has been counted: clear its counter for
+            // the next attention launch over the same plan
+            if (ct == 0)
+                p.unit_counter[pd.unit] = 0;
+        }
         pending = false;
         return true;
     };
+
+    // Trajectories without pages (n_b = 0, or a length outside [0, 16 * max_pages],
+    // which the planner reports) get out = 0 and lse = -inf here, each by one
+    // thread: trajectory b by CTA b % grid.  The planner writes the same rows; with
+    // this, every attention launch completes its own outputs, so one plan can serve
+    // several launches (the layers of one decode step).
+    {
+        const int max_len = p.max_pages * kPageSize;
+        const int ncand = ((int)blockIdx.x < p.batch)
+                              ? (p.batch - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x
+                              : 0;
+        for (int c = ct; c < ncand; c += kNumConsumerWarps * 32) {
+            const int b = (int)blockIdx.x + c * (int)gridDim.x;
+            const int n = p.context_lens[b];
+            if (n <= 0 || n > max_len) {
+                uint4 *row = reinterpret_cast<uint4 *>(p.out + (size_t)b * p.num_q_heads * D);
+                for (int v = 0; v < p.num_q_heads * D / 8; ++v)
+                    row[v] = make_uint4(0, 0, 0, 0);
+                if (p.lse)
+                    for (int h = 0; h < p.num_q_heads; ++h)
+                        p.lse[(size_t)b * p.num_q_heads + h] = -INFINITY;
+            }
+        }
+    }
 
     for (;;) {
         const uint32_t r = sc % kSegRing;

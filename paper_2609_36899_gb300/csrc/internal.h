@@ -71,7 +71,7 @@ struct alignas(64) WorkspaceHeader {
     int status;            // first device-side error code, 0 = none
     int slice_counter;     // next work slice to hand out
     int num_slices;        // T: slices of the flattened work sequence
-    int pad0;
+    int exit_counter;      // decode: CTAs done fetching slices (reset by the last one)
     long long total_work;  // W: page-heads (decode), copy units (staging), work units (prefill)
     long long total_items; // prefill: work items
     long long dp_items;    // prefill: items run whole (the rest are split)

@@ -208,6 +208,64 @@ def test_plan_then_run_equals_single_call():
     assert cadkv.decode_attention_status(ws) == 0
 
 
+def test_decode_step_matches_decode_attention():
+    """The binding's prepared call over fixed buffers gives decode_attention's
+    bits, call after call, as the inputs change in place."""
+    batch = make_batch([700, 12, 3300, 1], 16, 2, 128, seed=16)
+    q, k, v, bt, cl = device_tensors(batch)
+    out = torch.empty_like(q)
+    lse = torch.empty((4, 16), dtype=torch.float32, device="cuda")
+    ws = torch.empty(cadkv.decode_attention_workspace_size(4, 16, 2, 128, bt.shape[1]),
+                     dtype=torch.uint8, device="cuda")
+    step = cadkv.DecodeStep(q, k, v, bt, cl, out, lse, ws)
+    for i in range(2):
+        if i:
+            q.mul_(-0.5)                      # new values in the same buffers
+        ref_out, ref_lse = cadkv.decode_attention(q, k, v, bt, cl)
+        step()
+        torch.cuda.synchronize()
+        assert torch.equal(out, ref_out) and torch.equal(lse, ref_lse)
+
+
+@pytest.mark.parametrize("slice_pages", [0, 7])
+def test_plan_once_run_per_layer(slice_pages):
+    """One plan, then one run per layer (other q, pages and outputs, same
+    lengths), twice over: every run matches the oracle, including the rows of
+    an empty trajectory, which the planner never wrote for layers 1 and 2.
+    slice_pages = 7 forces more slices than CTAs, so every run hands slices out
+    through the counter the previous run put back."""
+    lens = [700, 0, 3300, 1, 45, 2048]
+    hq, hkv, d = 16, 2, 128
+    layers = [make_batch(lens, hq, hkv, d, seed=170 + l) for l in range(3)]  # own tables
+    cl = torch.from_numpy(layers[0].context_lens).cuda()
+    qs, ks, vs, bts, outs, lses, refs = [], [], [], [], [], [], []
+    for b in layers:
+        qs.append(b.q.cuda())
+        ks.append(b.k_pages.cuda())
+        vs.append(b.v_pages.cuda())
+        bts.append(torch.from_numpy(b.block_table).cuda())
+        outs.append(torch.full_like(qs[-1], float("nan")))
+        lses.append(torch.full((len(lens), hq), float("nan"), device="cuda"))
+        refs.append(oracle_decode(b))
+    width = bts[0].shape[1]
+    assert all(t.shape[1] == width for t in bts)
+    ws = torch.empty(cadkv.decode_attention_workspace_size(len(lens), hq, hkv, d, width),
+                     dtype=torch.uint8, device="cuda")
+    cadkv.decode_attention_plan(qs[0], ks[0], vs[0], bts[0], cl, outs[0], lses[0], ws,
+                                slice_pages=slice_pages)
+    for rnd in range(2):
+        for l in range(3):
+            if rnd:
+                outs[l].fill_(float("nan"))
+                lses[l].fill_(float("nan"))
+            cadkv.decode_attention_run(qs[l], ks[l], vs[l], bts[l], cl, outs[l], lses[l], ws)
+        torch.cuda.synchronize()
+        assert cadkv.decode_attention_status(ws) == 0
+        for l in range(3):
+            assert_close(outs[l], lses[l], refs[l][0], refs[l][1], f"round {rnd} layer {l}")
+            assert torch.all(outs[l][1] == 0) and torch.all(torch.isneginf(lses[l][1]))
+
+
 def test_status_reports_bad_page_without_faulting():
     batch = make_batch([40, 20], 4, 1, 64, seed=13, nan_tails=False)
     q, k, v, bt, cl = device_tensors(batch)
