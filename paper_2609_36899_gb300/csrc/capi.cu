@@ -200,7 +200,7 @@ struct AppendArgs {
 
 int plan_impl(const int32_t *context_lens, void *out, float *lse, const DecodeShape &s,
               int slice_pages, void *workspace, size_t workspace_bytes, cudaStream_t stream,
-              const AppendArgs *append = nullptr)
+              const AppendArgs *append = nullptr, bool describe_first = false)
 {
     int rc = check_decode_shape(s);
     if (rc != CADKV_OK)
@@ -228,6 +228,8 @@ int plan_impl(const int32_t *context_lens, void *out, float *lse, const DecodeSh
     p.hdr = reinterpret_cast<WorkspaceHeader *>(ws);
     p.page_prefix = reinterpret_cast<long long *>(ws + L.page_prefix);
     p.unit_counter = reinterpret_cast<int *>(ws + L.unit_counter);
+    p.first_seg = ws + L.first_seg;
+    p.describe_first = describe_first ? 1 : 0;
     p.batch = s.batch;
     p.num_q_heads = s.num_q_heads;
     p.num_kv_heads = s.num_kv_heads;
@@ -305,6 +307,7 @@ int run_impl(const void *q, const void *k_pages, const void *v_pages,
     p.lse = lse;
     p.hdr = reinterpret_cast<WorkspaceHeader *>(ws);
     p.page_prefix = reinterpret_cast<const long long *>(ws + L.page_prefix);
+    p.first_seg = ws + L.first_seg;
     p.unit_counter = reinterpret_cast<int *>(ws + L.unit_counter);
     p.part_lse = reinterpret_cast<float *>(ws + L.part_lse);
     p.part_o = reinterpret_cast<float *>(ws + L.part_o);
@@ -576,7 +579,7 @@ int decode_attention_plan(const int32_t *context_lens, void *out, float *lse, in
 {
     const DecodeShape s{batch, num_q_heads, num_kv_heads, head_dim, kPageSize, 1, max_pages};
     return plan_impl(context_lens, out, lse, s, slice_pages, workspace, workspace_bytes,
-                     reinterpret_cast<cudaStream_t>(stream));
+                     reinterpret_cast<cudaStream_t>(stream), nullptr, true);
 }
 
 int decode_attention_run(const void *q, const void *k_pages, const void *v_pages,

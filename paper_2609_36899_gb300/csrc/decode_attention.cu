@@ -49,6 +49,62 @@ constexpr float kLn2 = 0.6931471805599453f;
 
 __host__ __device__ constexpr size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// ------------------------------------------------------------------ work slices
+
+// One segment: the part of a (trajectory, KV head) unit inside one work slice.
+struct SegDesc {
+    int b, kvh, page_begin, num_pages;  // num_pages < 0: no more work
+    int n, slot, count, unit;
+    int first, pad[3];
+};
+
+// The planner's description of an attention CTA's first segment (slice i is
+// CTA i's first), so that the CTA starts streaming without working it out.
+struct FirstSeg {
+    SegDesc d;     // d.num_pages = 0: the slice is empty
+    long long s1;  // end of the slice
+    long long se;  // end of the segment: where the slice's next segment starts
+};
+static_assert(sizeof(FirstSeg) == kFirstSegBytes, "first-segment record size");
+
+__device__ __forceinline__ long long slice_begin(long long s, long long W, long long T)
+{
+    return s * W / T;
+}
+
+// Index of the slice containing flattened position x.
+__device__ __forceinline__ int slice_of(long long x, long long W, long long T)
+{
+    return (int)(((x + 1) * T + W - 1) / W - 1);
+}
+
+// The segment of slice `slice` (which ends at s1) that starts at flattened
+// position x inside trajectory b, whose page-heads are [pb0 * Hkv, pb1 * Hkv);
+// se receives where it ends.  d.n is left for the caller.
+__device__ __forceinline__ SegDesc describe_segment(long long x, int b, long long pb0, long long pb1,
+                                                    long long s1, int slice, long long W,
+                                                    long long T, int Hkv, long long &se)
+{
+    const long long pages_b = pb1 - pb0;
+    const long long base = pb0 * Hkv;
+    const int kvh = (int)((x - base) / pages_b);
+    const long long us = base + kvh * pages_b, ue = us + pages_b;
+    se = ue < s1 ? ue : s1;
+    const int first = slice_of(us, W, T), last = slice_of(ue - 1, W, T);
+    SegDesc d;
+    d.b = b;
+    d.kvh = kvh;
+    d.page_begin = (int)(x - us);
+    d.num_pages = (int)(se - x);
+    d.n = 0;
+    d.count = last - first + 1;
+    d.unit = b * Hkv + kvh;
+    d.slot = d.count == 1 ? -1 : d.unit + slice;
+    d.first = first;
+    d.pad[0] = d.pad[1] = d.pad[2] = 0;
+    return d;
+}
+
 // ------------------------------------------------------------------ planner
 
 // CTAs 1.. of the planner launch: write each trajectory's new-token K and V
@@ -100,6 +156,11 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(const PlanParams 
     }
     __shared__ long long warp_sums[32];
     __shared__ long long carry_s;
+    // small batches: the page prefix and clamped lengths also in shared memory,
+    // for describing the attention CTAs' first segments below
+    __shared__ long long s_prefix[kSmallPlanMaxBatch + 1];
+    __shared__ int s_len[kSmallPlanMaxBatch];
+    const bool small = p.describe_first && p.batch <= kSmallPlanMaxBatch;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int nthreads = blockDim.x, nwarps = nthreads >> 5;
     const int max_len = p.max_pages * kPageSize;
@@ -112,8 +173,9 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(const PlanParams 
     for (int base = 0; base < p.batch; base += nthreads) {
         const int b = base + tid;
         long long pages = 0;
+        int n = 0;
         if (b < p.batch) {
-            int n = p.context_lens[b];
+            n = p.context_lens[b];
             if (n < 0 || n > max_len) {
                 record_status(&p.hdr->status, CADKV_ERR_SHAPE);
                 n = 0;
@@ -153,8 +215,13 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(const PlanParams 
         __syncthreads();
         const long long carry = carry_s;
         const long long incl = carry + v + (warp > 0 ? warp_sums[warp - 1] : 0);
-        if (b < p.batch)
+        if (b < p.batch) {
             p.page_prefix[b] = incl - pages;
+            if (small) {
+                s_prefix[b] = incl - pages;
+                s_len[b] = n;  // the clamped length (0 when out of range)
+            }
+        }
         __syncthreads();
         if (tid == nthreads - 1)
             carry_s = incl;
@@ -162,28 +229,60 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(const PlanParams 
     }
     for (int i = tid; i < p.batch * p.num_kv_heads; i += nthreads)
         p.unit_counter[i] = 0;
+    const long long total = carry_s;
+    const int Hkv = p.num_kv_heads;
+    const long long W = total * Hkv;
+    // Dynamic slices (several per CTA) absorb per-SM speed differences, but
+    // each costs a start-up chain of dependent loads (slice, trajectory,
+    // table) and a pipeline fill; below ~4K page-heads per CTA that cost wins,
+    // so automatic slicing gives each CTA one equal slice there.
+    const long long T = plan_num_slices(W, p.slice_pages, p.slice_cap);
+    // Describe each attention CTA's first segment (its first slice is slice
+    // blockIdx.x), as its producer warp would: the CTA then loads one record
+    // instead of searching the prefix and dividing before its first copy.  This
+    // costs the planner about as much as it saves one attention launch, so only
+    // a plan made to serve several launches (decode_attention_plan) does it.
+    const long long ctas = p.slice_cap / kSlicesPerCta;
+    const long long nrec = small ? (T < ctas ? T : ctas) : 0;
+    if (small && tid == 0)
+        s_prefix[p.batch] = total;
+    __syncthreads();
+    for (long long i = tid; i < nrec; i += nthreads) {
+        FirstSeg f;
+        const long long s0 = slice_begin(i, W, T), s1 = slice_begin(i + 1, W, T);
+        f.s1 = s1;
+        if (s0 >= s1) {
+            f.d = SegDesc{};
+            f.d.num_pages = 0;
+            f.se = s0;
+        } else {
+            // largest b with s_prefix[b] <= s0 / Hkv (a trajectory with pages)
+            const long long v = s0 / Hkv;
+            int lo = 0, hi = p.batch - 1;
+            while (lo < hi) {
+                const int mid = (lo + hi + 1) >> 1;
+                if (s_prefix[mid] <= v)
+                    lo = mid;
+                else
+                    hi = mid - 1;
+            }
+            f.d = describe_segment(s0, lo, s_prefix[lo], s_prefix[lo + 1], s1, (int)i, W, T, Hkv,
+                                   f.se);
+            f.d.n = s_len[lo];
+        }
+        reinterpret_cast<FirstSeg *>(p.first_seg)[i] = f;
+    }
     if (tid == 0) {
-        const long long total = carry_s;
         p.page_prefix[p.batch] = total;
-        const long long W = total * p.num_kv_heads;
-        // Dynamic slices (several per CTA) absorb per-SM speed differences, but
-        // each costs a start-up chain of dependent loads (slice, trajectory,
-        // table) and a pipeline fill; below ~4K page-heads per CTA that cost wins,
-        // so automatic slicing gives each CTA one equal slice there.
         p.hdr->total_work = W;
-        p.hdr->num_slices = (int)plan_num_slices(W, p.slice_pages, p.slice_cap);
+        p.hdr->num_slices = (int)T;
         p.hdr->slice_counter = 0;
         p.hdr->exit_counter = 0;
+        p.hdr->first_segs = nrec;
     }
 }
 
 // ------------------------------------------------------------------ attention
-
-struct SegDesc {
-    int b, kvh, page_begin, num_pages;  // num_pages < 0: no more work
-    int n, slot, count, unit;
-    int first, pad[3];
-};
 
 template <int D>
 struct AttnConfig {
@@ -223,17 +322,6 @@ __device__ __forceinline__ int warp_find_trajectory(const long long *prefix, int
         hi = min(hi, lo + step - 1);
     }
     return lo;
-}
-
-__device__ __forceinline__ long long slice_begin(long long s, long long W, long long T)
-{
-    return s * W / T;
-}
-
-// Index of the slice containing flattened position x.
-__device__ __forceinline__ int slice_of(long long x, long long W, long long T)
-{
-    return (int)(((x + 1) * T + W - 1) / W - 1);
 }
 
 // All consumer threads (8 warps, 256 threads) arrive and wait; bounded, abort-aware.
@@ -323,6 +411,13 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         uint32_t kp = 0;  // page-heads issued
         uint32_t sp = 0;  // segments issued
         bool ok = true;
+        // The planner's description of this CTA's first segment, when it wrote one
+        // (small batches): the first copies then need no prefix search and no
+        // divisions here.
+        const bool have_rec = (long long)blockIdx.x < p.hdr->first_segs;
+        FirstSeg rec;
+        if (have_rec)
+            rec = reinterpret_cast<const FirstSeg *>(p.first_seg)[blockIdx.x];
         // Slice i < grid is CTA i's first; later slices come from the counter.
         int slice = blockIdx.x;
         for (bool initial = true; ok; initial = false) {
@@ -347,27 +442,46 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 }
                 break;
             }
-            const long long s0 = slice_begin(slice, W, T), s1 = slice_begin(slice + 1, W, T);
-            if (s0 >= s1)
-                continue;
-            int b = warp_find_trajectory(p.page_prefix, p.batch, s0 / Hkv, lane);
-            long long x = s0;
-            while (x < s1) {
-                const long long pb0 = p.page_prefix[b], pb1 = p.page_prefix[b + 1];
-                if (x >= pb1 * Hkv) {
-                    ++b;
+            bool use_rec = initial && have_rec;
+            long long x = 0, s1;
+            int b;
+            if (use_rec) {
+                if (rec.d.num_pages <= 0)
+                    continue;  // an empty slice
+                s1 = rec.s1;
+                b = rec.d.b;
+            } else {
+                const long long s0 = slice_begin(slice, W, T);
+                s1 = slice_begin(slice + 1, W, T);
+                if (s0 >= s1)
                     continue;
+                b = warp_find_trajectory(p.page_prefix, p.batch, s0 / Hkv, lane);
+                x = s0;
+            }
+            while (use_rec || x < s1) {
+                SegDesc d;
+                long long se;
+                int max_n = 0;  // > 0: d.n still to be read (and clamped to this)
+                if (use_rec) {
+                    d = rec.d;
+                    se = rec.se;
+                    use_rec = false;
+                } else {
+                    const long long pb0 = p.page_prefix[b], pb1 = p.page_prefix[b + 1];
+                    if (x >= pb1 * Hkv) {
+                        ++b;
+                        continue;
+                    }
+                    d = describe_segment(x, b, pb0, pb1, s1, slice, W, T, Hkv, se);
+                    max_n = (int)((pb1 - pb0) * kPageSize);
                 }
-                const long long pages_b = pb1 - pb0;
-                const long long base = pb0 * Hkv;
-                const int kvh = (int)((x - base) / pages_b);
-                const long long us = base + kvh * pages_b, ue = us + pages_b;
-                const int j0 = (int)(x - us);
-                const long long se = ue < s1 ? ue : s1;
-                const int npg = (int)(se - x);
-                const int first = slice_of(us, W, T), last = slice_of(ue - 1, W, T);
-                const int count = last - first + 1;
-                const int unit = b * Hkv + kvh;
+                const int npg = d.num_pages;
+                const int kvh = d.kvh;
+                const int *bt_row = p.block_table + (size_t)d.b * p.max_pages + d.page_begin;
+                // Block-table entries come 32 at a time, one chunk ahead of use; the
+                // first chunk's load is issued before the length's, so that the two
+                // latencies overlap.
+                int next_phys = lane < npg ? __ldg(bt_row + lane) : 0;
 
                 const uint32_t r = sp % kSegRing;
                 if (sp >= kSegRing) {
@@ -377,30 +491,18 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                         break;
                 }
                 if (lane == 0) {
-                    int n = p.context_lens[b];
-                    if (n > (int)(pages_b * kPageSize))
-                        n = (int)(pages_b * kPageSize);
-                    SegDesc d;
-                    d.b = b;
-                    d.kvh = kvh;
-                    d.page_begin = j0;
-                    d.num_pages = npg;
-                    d.n = n;
-                    d.slot = count == 1 ? -1 : unit + slice;
-                    d.count = count;
-                    d.unit = unit;
-                    d.first = first;
+                    if (max_n > 0) {
+                        const int n = p.context_lens[d.b];
+                        d.n = n < max_n ? n : max_n;
+                    }
                     desc[r] = d;
                     mbar_arrive_expect_tx(&seg_full[r], q_bytes);
                     bulk_load(qbuf + (size_t)r * kMaxGroup * D,
-                              p.q + ((size_t)b * p.num_q_heads + (size_t)kvh * G) * D, q_bytes,
+                              p.q + ((size_t)d.b * p.num_q_heads + (size_t)kvh * G) * D, q_bytes,
                               &seg_full[r]);
                 }
                 ++sp;
 
-                const int *bt_row = p.block_table + (size_t)b * p.max_pages + j0;
-                // Block-table entries come 32 at a time, one chunk ahead of use.
-                int next_phys = lane < npg ? __ldg(bt_row + lane) : 0;
                 for (int c = 0; c < npg && ok; c += 32) {
                     int phys = next_phys;
                     if (c + 32 + lane < npg)
@@ -845,6 +947,8 @@ DecodeWorkspaceLayout decode_workspace_layout(int batch, int num_kv_heads, int g
     size_t off = align_up(sizeof(WorkspaceHeader), kWorkspaceAlign);
     L.page_prefix = off;
     off = align_up(off + (size_t)(batch + 1) * sizeof(long long), kWorkspaceAlign);
+    L.first_seg = off;
+    off = align_up(off + (size_t)num_sms * kFirstSegBytes, kWorkspaceAlign);
     L.unit_counter = off;
     off = align_up(off + (size_t)batch * num_kv_heads * sizeof(int), kWorkspaceAlign);
     L.part_lse = off;

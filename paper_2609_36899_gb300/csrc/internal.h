@@ -76,12 +76,17 @@ struct alignas(64) WorkspaceHeader {
     long long total_items; // prefill: work items
     long long dp_items;    // prefill: items run whole (the rest are split)
     long long pieces;      // prefill: pieces per split item
-    long long pad1[2];
+    long long first_segs;  // decode: CTAs whose first segment the planner described (0: none)
+    long long pad1;
 };
 
 // Byte offsets of the decode-attention workspace regions.
+// Bytes of the planner's description of one attention CTA's first segment.
+constexpr size_t kFirstSegBytes = 64;
+
 struct DecodeWorkspaceLayout {
     size_t page_prefix;   // int64 [batch + 1]
+    size_t first_seg;     // kFirstSegBytes x #SM: each CTA's first segment, as planned
     size_t unit_counter;  // int32 [batch * Hkv]
     size_t part_lse;      // fp32  [capacity][G]
     size_t part_o;        // fp32  [capacity][G][D]
@@ -100,6 +105,8 @@ struct PlanParams {
     WorkspaceHeader *hdr;
     long long *page_prefix;
     int *unit_counter;
+    void *first_seg;    // [slice_cap / kSlicesPerCta] first-segment records
+    int describe_first; // 1: write them (a plan that may serve several runs)
     int batch, num_q_heads, num_kv_heads, head_dim, max_pages;
     int slice_cap;      // upper bound on slices (partial capacity)
     int slice_pages;    // forced slice length in pages, 0 = automatic
@@ -125,6 +132,7 @@ struct AttnParams {
     float *lse;
     WorkspaceHeader *hdr;
     const long long *page_prefix;
+    const void *first_seg;  // the planner's first-segment records (valid: hdr->first_segs)
     int *unit_counter;
     float *part_lse;
     float *part_o;

@@ -60,6 +60,29 @@ def test_full_size_every_row(w):
     torch.cuda.empty_cache()
 
 
+def test_mixed_full_size_plan_then_run_bit_identical():
+    """The bench's headline launches (decode_attention_plan, whose planner also
+    describes every attention CTA's first segment, then decode_attention_run) give
+    the same bits as decode_attention, whose CTAs work their first segment out
+    themselves, on the full-size mixed batch; the latter is checked against the
+    oracle on every row above."""
+    batch = make_decode_batch(MIXED, device="cuda")
+    q, k, v = batch.q, batch.k_pages, batch.v_pages
+    bt = torch.from_numpy(batch.block_table).cuda()
+    cl = torch.from_numpy(batch.context_lens).cuda()
+    out, lse = cadkv.decode_attention(q, k, v, bt, cl)
+    out2, lse2 = torch.empty_like(out), torch.empty_like(lse)
+    ws = torch.empty(cadkv.decode_attention_workspace_size(MIXED.batch, 64, 8, 128, bt.shape[1]),
+                     dtype=torch.uint8, device="cuda")
+    cadkv.decode_attention_plan(q, k, v, bt, cl, out2, lse2, ws)
+    cadkv.decode_attention_run(q, k, v, bt, cl, out2, lse2, ws)
+    torch.cuda.synchronize()
+    assert cadkv.decode_attention_status(ws) == 0
+    assert torch.equal(out, out2) and torch.equal(lse, lse2)
+    del batch, q, k, v
+    torch.cuda.empty_cache()
+
+
 @pytest.mark.parametrize("slice_pages", [61, 4096, 1 << 20])
 def test_mixed_full_size_forced_slices_every_row(slice_pages):
     """The full-size mixed batch with the work slices forced short (many
