@@ -248,15 +248,30 @@ def test_decode_step_matches_decode_attention():
         step()
         torch.cuda.synchronize()
         assert torch.equal(out, ref_out) and torch.equal(lse, ref_lse)
+    # one prepared plan, then prepared runs over two layers' pages
+    k2, v2 = torch.flip(k, dims=[0]), torch.flip(v, dims=[0])
+    bt2 = (k.shape[0] - 1 - bt).where(bt >= 0, bt)   # the same logical pages, moved
+    plan = cadkv.DecodeStep(q, k, v, bt, cl, out, lse, ws, launch="plan")
+    runs = [cadkv.DecodeStep(q, k, v, bt, cl, out, lse, ws, launch="run"),
+            cadkv.DecodeStep(q, k2, v2, bt2, cl, out, lse, ws, launch="run")]
+    ref_out, ref_lse = cadkv.decode_attention(q, k, v, bt, cl)
+    plan()
+    for run in runs + runs:
+        out.fill_(float("nan"))
+        run()
+        torch.cuda.synchronize()
+        assert torch.equal(out, ref_out) and torch.equal(lse, ref_lse)
 
 
-@pytest.mark.parametrize("slice_pages", [0, 7])
+@pytest.mark.parametrize("slice_pages", [0, 7, 3, 1])
 def test_plan_once_run_per_layer(slice_pages):
     """One plan, then one run per layer (other q, pages and outputs, same
     lengths), twice over: every run matches the oracle, including the rows of
     an empty trajectory, which the planner never wrote for layers 1 and 2.
-    slice_pages = 7 forces more slices than CTAs, so every run hands slices out
-    through the counter the previous run put back."""
+    The batch has 766 page-heads: slice_pages = 3 and 1 cut 256 and 608 slices,
+    more than the CTAs, so every run hands slices out through the counter the
+    previous run put back, and merges many partials through arrival counters
+    the previous run cleared."""
     lens = [700, 0, 3300, 1, 45, 2048]
     hq, hkv, d = 16, 2, 128
     layers = [make_batch(lens, hq, hkv, d, seed=170 + l) for l in range(3)]  # own tables
