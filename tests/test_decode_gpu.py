@@ -99,6 +99,22 @@ def test_mixed_full_size_forced_slices_every_row(slice_pages):
     torch.cuda.empty_cache()
 
 
+@pytest.mark.parametrize("slice_pages", [0, 5])
+@pytest.mark.parametrize("hq,hkv,d", [(16, 2, 64), (40, 8, 128)], ids=["G8-D64", "G5-D128"])
+def test_mid_size_heavy_tailed_every_row(hq, hkv, d, slice_pages):
+    """A mid-size heavy-tailed batch, 300 trajectories with lengths lognormal
+    (median 600) clipped to [1, 20,000], for head_dim 64 (the 32-stage ring of
+    4 KB stages) and for Qwen3-14B's 40/8 heads (G = 5, three padded query rows
+    per MMA tile); automatic slicing and forced short slices (dynamic, many
+    partials); every row against the oracle."""
+    rng = np.random.Generator(np.random.PCG64(640))
+    lens = np.clip(np.round(600 * np.exp(rng.normal(0, 1.2, 300))), 1, 20000).astype(np.int32)
+    batch = make_batch(lens, hq, hkv, d, seed=641 + d)
+    out, lse = gpu_decode(batch, slice_pages=slice_pages)
+    ref, ref_lse = oracle_decode(batch)
+    assert_close(out, lse, ref, ref_lse, f"{hq}/{hkv} heads D={d}, slice_pages={slice_pages}")
+
+
 @pytest.mark.parametrize("g,d", [(1, 64), (2, 128), (4, 64), (8, 128), (8, 64), (3, 128),
                                  (5, 128)])
 def test_edge_lengths(g, d):
