@@ -307,16 +307,16 @@ def test_plan_once_run_per_layer(slice_pages):
                      dtype=torch.uint8, device="cuda")
     cadkv.decode_attention_plan(qs[0], ks[0], vs[0], bts[0], cl, outs[0], lses[0], ws,
                                 slice_pages=slice_pages)
-    for rnd in range(2):
+    for pass_ in range(2):
         for l in range(3):
-            if rnd:
+            if pass_:
                 outs[l].fill_(float("nan"))
                 lses[l].fill_(float("nan"))
             cadkv.decode_attention_run(qs[l], ks[l], vs[l], bts[l], cl, outs[l], lses[l], ws)
         torch.cuda.synchronize()
         assert cadkv.decode_attention_status(ws) == 0
         for l in range(3):
-            assert_close(outs[l], lses[l], refs[l][0], refs[l][1], f"round {rnd} layer {l}")
+            assert_close(outs[l], lses[l], refs[l][0], refs[l][1], f"pass {pass_} layer {l}")
             assert torch.all(outs[l][1] == 0) and torch.all(torch.isneginf(lses[l][1]))
 
 
