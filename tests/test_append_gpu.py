@@ -50,6 +50,31 @@ def test_append_then_attend(g, d):
     assert_close(out, lse, ref, ref_lse, f"append G={g} D={d}")
 
 
+def test_append_large_batch():
+    """3,000 trajectories x 4 KV heads: 375 append CTAs beside the 1,024-thread
+    planner.  The pool after the append equals the oracle's kv_append, and the
+    attention over it matches the oracle on every row."""
+    rng = np.random.Generator(np.random.PCG64(330))
+    lens = rng.integers(0, 300, 3000).astype(np.int32)
+    batch = make_batch(lens, 16, 4, 64, seed=331)
+    k_new, v_new = _new_rows(3000, 4, 64, seed=332)
+    kp = bf16_bits(batch.k_pages).copy()
+    vp = bf16_bits(batch.v_pages).copy()
+    oracle.kv_append(kp, vp, bf16_bits(k_new), bf16_bits(v_new), batch.block_table,
+                     batch.context_lens)
+    q = batch.q.cuda()
+    k_dev, v_dev = batch.k_pages.cuda(), batch.v_pages.cuda()
+    bt = torch.from_numpy(batch.block_table).cuda()
+    cl = torch.from_numpy(batch.context_lens).cuda()
+    out, lse = cadkv.decode_attention_append(q, k_new.cuda(), v_new.cuda(), k_dev, v_dev, bt, cl)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(bf16_bits(k_dev), kp)
+    np.testing.assert_array_equal(bf16_bits(v_dev), vp)
+    ref, ref_lse = oracle.decode_attention(bf16_bits(batch.q), kp, vp, batch.block_table,
+                                           batch.context_lens)
+    assert_close(out, lse, ref, ref_lse, "append, B = 3000")
+
+
 def test_append_full_size_mixed_every_row():
     """The whole decode step of the full-size mixed batch (512 trajectories,
     dynamic-slice path).  The pool after the append equals the oracle's

@@ -99,6 +99,30 @@ def test_mixed_full_size_forced_slices_every_row(slice_pages):
     torch.cuda.empty_cache()
 
 
+@pytest.mark.parametrize("slice_pages", [0, 3])
+def test_large_batch_every_row(slice_pages):
+    """6,000 trajectories (above the batch size up to which a 256-thread planner
+    runs and describes the CTAs' first segments: here the 1,024-thread planner
+    scans the lengths in six rounds), lengths U[0, 600] with some empty, 8/2
+    heads, D = 64; automatic and forced short slices; every row against the
+    oracle, through the planner and attention launches separately as well."""
+    rng = np.random.Generator(np.random.PCG64(660))
+    lens = rng.integers(0, 601, 6000).astype(np.int32)
+    lens[::97] = 0
+    batch = make_batch(lens, 8, 2, 64, seed=661)
+    q, k, v, bt, cl = device_tensors(batch)
+    out, lse = gpu_decode(batch, slice_pages=slice_pages, tensors=(q, k, v, bt, cl))
+    ref, ref_lse = oracle_decode(batch)
+    assert_close(out, lse, ref, ref_lse, f"B=6000, slice_pages={slice_pages}")
+    out2, lse2 = torch.empty_like(out), torch.empty_like(lse)
+    ws = torch.empty(cadkv.decode_attention_workspace_size(6000, 8, 2, 64, bt.shape[1]),
+                     dtype=torch.uint8, device="cuda")
+    cadkv.decode_attention_plan(q, k, v, bt, cl, out2, lse2, ws, slice_pages=slice_pages)
+    cadkv.decode_attention_run(q, k, v, bt, cl, out2, lse2, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(out, out2) and torch.equal(lse, lse2)
+
+
 @pytest.mark.parametrize("slice_pages", [0, 5])
 @pytest.mark.parametrize("hq,hkv,d", [(16, 2, 64), (40, 8, 128)], ids=["G8-D64", "G5-D128"])
 def test_mid_size_heavy_tailed_every_row(hq, hkv, d, slice_pages):
