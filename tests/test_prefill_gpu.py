@@ -60,6 +60,20 @@ def test_prefill_many_tiles():
     assert_close(out, lse, ref, ref_lse, "prefill many tiles")
 
 
+def test_prefill_many_trajectories():
+    """1,500 trajectories (the 1,024-thread planner scans their work items in two
+    rounds), contexts U[1, 400], chunks of 1..24 tokens: many small items, with
+    the last partial wave split; every row against the oracle."""
+    rng = np.random.Generator(np.random.PCG64(430))
+    lens = rng.integers(1, 401, 1500)
+    chunks = np.minimum(lens, rng.integers(1, 25, 1500))
+    batch, offs, q = _case(lens.tolist(), chunks.tolist(), 8, 2, seed=431)
+    out, lse, ws = _run(batch, offs, q)
+    assert cadkv.prefill_attention_status(ws) == 0
+    ref, ref_lse = _oracle(batch, offs, q)
+    assert_close(out, lse, ref, ref_lse, "prefill, 1,500 trajectories")
+
+
 def test_prefill_qwen_shape():
     """32 query / 8 KV heads (G = 4), contexts of a few thousand tokens."""
     lens, chunks = [3000, 4500], [256, 130]

@@ -66,6 +66,34 @@ def test_stage_bit_exact(d, lb, le):
     assert np.all(got[size:] == 0x1234)
 
 
+def test_stage_and_load_many_trajectories():
+    """1,500 trajectories (the planner's prefix sums run over several 1,024-wide
+    rounds), lengths 0..200, 2 layers: staging bit-exact against the oracle, and
+    loading the rows back into a cleared pool restores every used slot."""
+    rng = np.random.Generator(np.random.PCG64(31))
+    lens = rng.integers(0, 201, 1500)
+    lens, table, kp, vp = make_case(lens.tolist(), 2, 2, 64, seed=32)
+    pool, k_layers, v_layers = to_pool(kp, vp)
+    bt, cl = torch.from_numpy(table).cuda(), torch.from_numpy(lens).cuda()
+    size = cadkv.staged_size(lens, 0, 2, 2, 64)
+    dst = torch.empty(size, dtype=torch.bfloat16, device="cuda")
+    ws = cadkv.kv_prefix_stage(pool, bt, cl, 0, 2, dst)
+    assert cadkv.kv_prefix_stage_status(ws) == 0
+    np.testing.assert_array_equal(bf16_bits(dst), oracle_stage(kp, vp, table, lens, 0, 2))
+    for t in k_layers + v_layers:
+        t.view(torch.int16).fill_(0)
+    cadkv.kv_prefix_load(pool, bt, cl, 0, 2, dst, workspace=ws)
+    assert cadkv.kv_prefix_stage_status(ws) == 0
+    kz = torch.zeros_like(kp)
+    vz = torch.zeros_like(vp)
+    kl, vl = oracle.prefix_load(bf16_bits(kz.reshape(-1)).reshape(kz.shape).copy(),
+                                bf16_bits(vz.reshape(-1)).reshape(vz.shape).copy(),
+                                table, lens, 0, 2, bf16_bits(dst))
+    for l in range(2):
+        np.testing.assert_array_equal(bf16_bits(k_layers[l]), kl[l])
+        np.testing.assert_array_equal(bf16_bits(v_layers[l]), vl[l])
+
+
 def test_stage_explicit_offsets_keep_gaps():
     lens, table, kp, vp = make_case([9, 33, 1], 2, 2, 128, seed=21)
     pool, _, _ = to_pool(kp, vp)
