@@ -376,14 +376,24 @@ int cadkv_hbm_read_probe(const void *buf, size_t bytes, unsigned long long *sink
  *   (status word, work counter, arrival counters) itself.  Calls whose
  *   kernels may overlap on the GPU (different streams without ordering) race
  *   on the array and give wrong results: order them on one stream.
- * - The device status word of the last call is not exposed by this entry
- *   point; use decode_attention with a workspace when it is needed.
+ * - The device status word of the last call (bad block-table entries, lengths
+ *   beyond the table, timeouts) is read by decode_attention_noalloc_status.
  */
 int decode_attention_noalloc(const void *q, const void *k_pages, const void *v_pages,
                              const int32_t *block_table, const int32_t *context_lens,
                              void *out, float *lse, int batch, int num_q_heads,
                              int num_kv_heads, int head_dim, int page_size, int num_pages,
                              int max_pages, cadkv_stream_t stream);
+
+/*
+ * Device status word of the last decode_attention_noalloc call on the current
+ * device's context, as decode_attention_status reads it from a workspace:
+ * synchronises `stream` (pass the stream of that call), returns 0 or the first
+ * CADKV_ERR_* the kernels recorded (CADKV_ERR_OOB, CADKV_ERR_SHAPE,
+ * CADKV_ERR_TIMEOUT), or CADKV_ERR_CUDA if the copy fails.  The next call
+ * clears the word, so read it before calling again.
+ */
+int decode_attention_noalloc_status(cadkv_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -13,7 +13,7 @@ for sm_103a, C ABI in ``include/cadkv.h``).  Build it with
 from ._binding import (  # noqa: F401
     STATUS, CadkvError, DecodeStep, KVPool, LibraryMissing, cadkv_hbm_read_probe, cadkv_wait_selftest,
     decode_attention,
-    decode_attention_append, decode_attention_noalloc, decode_attention_plan, decode_attention_run, decode_attention_status,
+    decode_attention_append, decode_attention_noalloc, decode_attention_noalloc_status, decode_attention_plan, decode_attention_run, decode_attention_status,
     decode_attention_workspace_size, header_functions, kv_prefix_load,
     kv_prefix_stage, kv_prefix_stage_status, kv_prefix_stage_workspace_size,
     kv_status_string, library, prefill_attention, prefill_attention_status, staged_size,

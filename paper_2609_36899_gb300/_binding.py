@@ -61,6 +61,7 @@ _SIGNATURES = {
                                      _I, _I, _P, _SZ, _P]),
     "decode_attention_noalloc": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I,
                                       _P]),
+    "decode_attention_noalloc_status": (_I, [_P]),
     "kv_prefix_stage_workspace_size": (_SZ, [_I]),
     "kv_prefix_stage": (_I, [_P, _P, _I, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
     "kv_prefix_load": (_I, [_P, _P, _I, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
@@ -312,6 +313,13 @@ def decode_attention_noalloc(q, k_pages, v_pages, block_table, context_lens, out
         _stream(stream, q.device))
     _check("decode_attention_noalloc", rc)
     return out, lse
+
+
+def decode_attention_noalloc_status(stream=None, device=None) -> int:
+    """Synchronise the stream and return the status word of the last
+    decode_attention_noalloc call on the device (0 = ok)."""
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else device
+    return int(library().decode_attention_noalloc_status(_stream(stream, dev)))
 
 
 def prefill_attention(q, q_offsets, k_pages, v_pages, block_table, context_lens, out=None,

@@ -24,7 +24,7 @@ struct cadkv_pool {
 
 namespace {
 
-constexpr int kAbiVersion = (1 << 16) | 1;
+constexpr int kAbiVersion = (1 << 16) | 2;
 
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
@@ -872,6 +872,16 @@ int decode_attention_noalloc(const void *q, const void *k_pages, const void *v_p
         return rc;
     return run_impl(q, k_pages, v_pages, block_table, context_lens, out, lse, s, scratch,
                     CADKV_NOALLOC_SCRATCH_BYTES, st);
+}
+
+int decode_attention_noalloc_status(cadkv_stream_t stream)
+{
+    void *scratch = nullptr;
+    const int rc = noalloc_scratch(&scratch);
+    if (rc != CADKV_OK)
+        return rc;
+    // the status word is the first field of the workspace header at the array's start
+    return read_status(scratch, reinterpret_cast<cudaStream_t>(stream));
 }
 
 size_t kv_prefix_stage_workspace_size(int batch)

@@ -153,3 +153,38 @@ def test_noalloc_rejects_problems_beyond_the_scratch():
     assert _call_noalloc(q, k, k, bt, cl, out, lse) == STATUS["CADKV_ERR_WORKSPACE"]
     torch.cuda.synchronize()
     assert torch.all(out == 7.0)   # nothing ran
+
+
+def test_noalloc_status_reports_bad_input_without_faulting():
+    """The status word of the last call, read through the C ABI: a block-table
+    entry outside the pool is read as page 0 and flagged CADKV_ERR_OOB, a length
+    beyond the table is treated as empty and flagged CADKV_ERR_SHAPE, and the
+    next good call clears the word.  The untouched trajectories still match the
+    oracle."""
+    lib = cadkv.library()
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    q, k, v, bt, cl = _inputs([40, 20, 300], 8, 2, 64, seed=21)
+    out = torch.empty_like(q)
+    lse = torch.empty((3, 8), dtype=torch.float32, device="cuda")
+    assert _call_noalloc(q, k, v, bt, cl, out, lse) == 0
+    assert lib.decode_attention_noalloc_status(stream) == 0
+
+    good = int(bt[1, 0])
+    bt[1, 0] = k.shape[0] + 5                       # outside the pool
+    assert _call_noalloc(q, k, v, bt, cl, out, lse) == 0
+    assert lib.decode_attention_noalloc_status(stream) == STATUS["CADKV_ERR_OOB"]
+    keep = torch.tensor([0, 2], device="cuda")
+    _compare_oracle(out[keep], lse[keep], q[keep], k, v, bt[keep], cl[keep])
+    bt[1, 0] = good
+
+    cl[1] = bt.shape[1] * 16 + 1                    # longer than its table row
+    assert _call_noalloc(q, k, v, bt, cl, out, lse) == 0
+    assert lib.decode_attention_noalloc_status(stream) == STATUS["CADKV_ERR_SHAPE"]
+    assert torch.all(out[1] == 0) and torch.all(torch.isneginf(lse[1]))
+    cl[1] = 20
+
+    assert _call_noalloc(q, k, v, bt, cl, out, lse) == 0
+    assert lib.decode_attention_noalloc_status(stream) == 0
+    _compare_oracle(out, lse, q, k, v, bt, cl)
+    # the binding's accessor reads the same word
+    assert cadkv.decode_attention_noalloc_status() == 0
