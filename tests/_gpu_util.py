@@ -50,14 +50,51 @@ def assert_close(out_gpu, lse_gpu, out_ref, lse_ref, what=""):
     err = np.abs(o - out_ref).max(initial=0.0)
     assert err <= OUT_ATOL, f"{what}: max |out err| = {err:.3e} > {OUT_ATOL}"
     if lse_gpu is not None:
-        l = lse_gpu.cpu().numpy().astype(np.float64).reshape(lse_ref.shape)
-        inf_ref = np.isneginf(lse_ref)
-        assert np.array_equal(np.isneginf(l), inf_ref), f"{what}: -inf lse mismatch"
-        fin = ~inf_ref
-        if fin.any():
-            rel = np.abs(l[fin] - lse_ref[fin]) / np.maximum(np.abs(lse_ref[fin]), 1.0)
-            assert rel.max() <= LSE_RTOL, f"{what}: max lse rel err = {rel.max():.3e}"
+        _assert_lse(lse_gpu, lse_ref, what)
     return err
+
+
+def _assert_lse(lse_gpu, lse_ref, what):
+    l = lse_gpu.cpu().numpy().astype(np.float64).reshape(lse_ref.shape)
+    inf_ref = np.isneginf(lse_ref)
+    assert np.array_equal(np.isneginf(l), inf_ref), f"{what}: -inf lse mismatch"
+    fin = ~inf_ref
+    if fin.any():
+        rel = np.abs(l[fin] - lse_ref[fin]) / np.maximum(np.abs(lse_ref[fin]), 1.0)
+        assert rel.max() <= LSE_RTOL, f"{what}: max lse rel err = {rel.max():.3e}"
+
+
+U_BF16 = 2.0 ** -8   # unit roundoff of bf16 (8-bit significand)
+
+
+def abs_bits(bits: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns with the sign bit cleared: |x| (NaN stays NaN)."""
+    return bits & np.uint16(0x7FFF)
+
+
+def assert_close_bounded(out_gpu, lse_gpu, out_ref, lse_ref, absv_ref, what=""):
+    """assert_close with each output element's bound raised to what the
+    arithmetic itself guarantees, where that is larger than 1e-2.
+
+    Both kernels round the softmax weights P to bf16 before the P.V product
+    (tensor-core operands have one type, and V is bf16) and round out to bf16;
+    the row sum comes from the unrounded P.  With u = 2^-8 and w_j the exact
+    weights, out_gpu = (1 + e)(sum_j w_j (1 + d_j) v_j) with |d_j|, |e| <= u, so
+    |out_gpu - out_ref| <= u (sum_j w_j |v_j| + |out_ref|) up to fp32 rounding.
+    `absv_ref` is sum_j w_j |v_j| per element: the oracle run on |V|.  Rows over
+    many keys stay at 1e-2 (the bound is ~3e-3 there); a row over a handful of
+    keys whose values are large (|v| ~ 4) can reach ~1.5e-2, and gets the bound.
+    """
+    o = out_gpu.float().cpu().numpy().astype(np.float64).reshape(out_ref.shape)
+    assert np.all(np.isfinite(o)), f"{what}: non-finite output"
+    bound = U_BF16 * (absv_ref + np.abs(out_ref)) * 1.01 + 1e-4
+    tol = np.maximum(OUT_ATOL, bound)
+    excess = np.abs(o - out_ref) - tol
+    worst = np.unravel_index(np.argmax(excess), excess.shape)
+    assert excess[worst] <= 0, (f"{what}: |out err| {abs(o - out_ref)[worst]:.3e} > "
+                                f"bound {tol[worst]:.3e} at {tuple(int(i) for i in worst)}")
+    if lse_gpu is not None:
+        _assert_lse(lse_gpu, lse_ref, what)
 
 
 def make_batch(lens, hq, hkv, d, seed, extra_pages=5, max_pages=None, nan_tails=True,
