@@ -738,8 +738,8 @@ def _decode_cell(w, device, steps, warmup):
     return cell
 
 
-def bench_landscape(device, steps, warmup, batches=(8, 32, 128, 512),
-                    means=(1024, 4096, 16384, 65536), max_tokens=8 << 20):
+def bench_landscape(device, steps, warmup, batches=(8, 32, 128, 512, 2048),
+                    means=(256, 1024, 4096, 16384, 65536), max_tokens=8 << 20):
     """Decode GB/s and steps/s over (B, mean context), 32/8 heads, D = 128."""
     cells = []
     for b in batches:

@@ -87,10 +87,14 @@ __device__ __forceinline__ SegDesc describe_segment(long long x, int b, long lon
 {
     const long long pages_b = pb1 - pb0;
     const long long base = pb0 * Hkv;
-    const int kvh = (int)((x - base) / pages_b);
+    const long long rel = x - base;
+    const int kvh = rel <= 0xffffffffLL ? (int)((unsigned)rel / (unsigned)pages_b)
+                                        : (int)(rel / pages_b);
     const long long us = base + kvh * pages_b, ue = us + pages_b;
     se = ue < s1 ? ue : s1;
-    const int first = slice_of(us, W, T), last = slice_of(ue - 1, W, T);
+    // x lies in slice `slice`: a unit that starts at x, or ends by s1, needs no search
+    const int first = us == x ? slice : slice_of(us, W, T);
+    const int last = ue <= s1 ? slice : slice_of(ue - 1, W, T);
     SegDesc d;
     d.b = b;
     d.kvh = kvh;
@@ -236,14 +240,20 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(const PlanParams 
     // each costs a start-up chain of dependent loads (slice, trajectory,
     // table) and a pipeline fill; below ~4K page-heads per CTA that cost wins,
     // so automatic slicing gives each CTA one equal slice there.
-    const long long T = plan_num_slices(W, p.slice_pages, p.slice_cap);
+    const long long ctas = p.slice_cap / kSlicesPerCta;
+    // Short units (automatic slicing only): one slice per consumer warp, each
+    // warp on its own (see kWarpModeMaxAvgPages).
+    const long long units = (long long)p.batch * Hkv;
+    const long long warp_slices = ctas * kNumConsumerWarps;
+    const bool warp_mode = p.slice_pages == 0 && W <= kWarpModeMaxAvgPages * units &&
+                           W >= kWarpModeMinSlicePages * warp_slices;
+    const long long T = warp_mode ? warp_slices : plan_num_slices(W, p.slice_pages, p.slice_cap);
     // Describe each attention CTA's first segment (its first slice is slice
     // blockIdx.x), as its producer warp would: the CTA then loads one record
     // instead of searching the prefix and dividing before its first copy.  This
     // costs the planner about as much as it saves one attention launch, so only
     // a plan made to serve several launches (decode_attention_plan) does it.
-    const long long ctas = p.slice_cap / kSlicesPerCta;
-    const long long nrec = small ? (T < ctas ? T : ctas) : 0;
+    const long long nrec = small && !warp_mode ? (T < ctas ? T : ctas) : 0;
     if (small && tid == 0)
         s_prefix[p.batch] = total;
     __syncthreads();
@@ -279,6 +289,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(const PlanParams 
         p.hdr->slice_counter = 0;
         p.hdr->exit_counter = 0;
         p.hdr->first_segs = nrec;
+        p.hdr->warp_mode = warp_mode ? 1 : 0;
     }
 }
 
@@ -304,6 +315,101 @@ struct AttnConfig {
     static constexpr size_t kFlagOff = kBarOff + (size_t)kNumBars * 8;
     static constexpr size_t kBytes = kFlagOff + 16 + 1024;  // + slack for 1024-B alignment
 };
+
+// One page-head of a segment for one warp: S^T = K Q^T (16 tokens x 8 query
+// heads, mma.sync m16n8k16), online softmax over the page's valid tokens, and
+// O^T += V^T P^T.  kbase: the stage's K block (V follows it); tokens at or past
+// `valid` are masked and their V rows zeroed (they may hold NaN).
+template <int D>
+__device__ __forceinline__ void attend_page(uint32_t kbase, int valid,
+                                            const uint32_t (&qf)[D / 16][2], float scale_log2,
+                                            float &m0, float &m1, float &l0, float &l1,
+                                            float (&o)[D / 16][4], int lane)
+{
+    using C = AttnConfig<D>;
+    const int g = lane >> 2, t = lane & 3;    // mma fragment coordinates
+    const int mi = lane >> 3, rr = lane & 7;  // ldmatrix: matrix index, row in matrix
+    const uint32_t vbase = kbase + C::kKBytes;
+
+    // ---- S^T (16 tokens x 8 heads) = K (16 x D) . Q^T (D x 8)
+    float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
+    {
+        const int row = (mi & 1) * 8 + rr;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+            const int chunk = 2 * kk + (mi >> 1);
+            const uint32_t addr = kbase + (chunk >> 3) * C::kBoxBytes + row * 128 +
+                                  (((chunk & 7) ^ rr) << 4);
+            uint32_t a0, a1, a2, a3;
+            ldmatrix_x4(addr, a0, a1, a2, a3);
+            if (kk & 1)
+                mma_bf16_m16n8k16(sb, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
+            else
+                mma_bf16_m16n8k16(sa, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
+        }
+    }
+    // s[0]: (token g, head 2t)  s[1]: (g, 2t+1)  s[2]: (g+8, 2t)  s[3]: (g+8, 2t+1)
+    float s[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+        s[e] = (sa[e] + sb[e]) * scale_log2;
+    if (valid < kPageSize) {
+        if (g >= valid) {
+            s[0] = -INFINITY;
+            s[1] = -INFINITY;
+        }
+        if (g + 8 >= valid) {
+            s[2] = -INFINITY;
+            s[3] = -INFINITY;
+        }
+    }
+    float mx0 = fmaxf(s[0], s[2]), mx1 = fmaxf(s[1], s[3]);
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+        mx0 = fmaxf(mx0, __shfl_xor_sync(kFull, mx0, off));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(kFull, mx1, off));
+    }
+    const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+    const float alpha0 = exp2_approx(m0 - mn0), alpha1 = exp2_approx(m1 - mn1);
+    m0 = mn0;
+    m1 = mn1;
+    const float p0 = exp2_approx(s[0] - mn0), p1 = exp2_approx(s[1] - mn1);
+    const float p2 = exp2_approx(s[2] - mn0), p3 = exp2_approx(s[3] - mn1);
+    l0 = l0 * alpha0 + (p0 + p2);
+    l1 = l1 * alpha1 + (p1 + p3);
+#pragma unroll
+    for (int mt = 0; mt < D / 16; ++mt) {
+        o[mt][0] *= alpha0;
+        o[mt][1] *= alpha1;
+        o[mt][2] *= alpha0;
+        o[mt][3] *= alpha1;
+    }
+    // P^T as the B operand: transpose the two 8x8 (token x head) blocks.
+    const uint32_t pb0 = movmatrix_trans(pack_bf16x2(p0, p1));
+    const uint32_t pb1 = movmatrix_trans(pack_bf16x2(p2, p3));
+    uint32_t mask_lo = 0xffffffffu, mask_hi = 0xffffffffu;
+    if (valid < kPageSize) {  // zero value rows past n (they may hold NaN)
+        mask_lo = (2 * t < valid ? 0x0000ffffu : 0u) | (2 * t + 1 < valid ? 0xffff0000u : 0u);
+        mask_hi = (2 * t + 8 < valid ? 0x0000ffffu : 0u) | (2 * t + 9 < valid ? 0xffff0000u : 0u);
+    }
+    // ---- O^T (D x 8) += V^T (D x 16 tokens) . P^T (16 x 8)
+    {
+        const int row = (mi >> 1) * 8 + rr;
+#pragma unroll
+        for (int mt = 0; mt < D / 16; ++mt) {
+            const int chunk = 2 * mt + (mi & 1);
+            const uint32_t addr = vbase + (chunk >> 3) * C::kBoxBytes + row * 128 +
+                                  (((chunk & 7) ^ rr) << 4);
+            uint32_t a0, a1, a2, a3;
+            ldmatrix_x4_trans(addr, a0, a1, a2, a3);
+            a0 &= mask_lo;
+            a1 &= mask_lo;
+            a2 &= mask_hi;
+            a3 &= mask_hi;
+            mma_bf16_m16n8k16(o[mt], a0, a1, a2, a3, pb0, pb1);
+        }
+    }
+}
 
 // Largest b in [0, batch) with prefix[b] <= v, given prefix non-decreasing,
 // prefix[0] = 0 <= v < prefix[batch].  Whole warp cooperates (32-way search).
@@ -399,9 +505,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
     const long long W = p.hdr->total_work;
     const int T = p.hdr->num_slices;
+    const bool warp_mode = p.hdr->warp_mode != 0;
 
     if (warp == kNumConsumerWarps) {
         // ============================ producer warp ============================
+        if (warp_mode)  // every consumer warp loads its own pages
+            return;
         if (lane == 0) {
             prefetch_tensor_map(&kmap);
             prefetch_tensor_map(&vmap);
@@ -600,7 +709,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
     // ================================ consumer warps ================================
     const int g = lane >> 2, t = lane & 3;          // mma fragment coordinates
-    const int mi = lane >> 3, rr = lane & 7;        // ldmatrix: matrix index, row in matrix
     const int ct = tid;                             // consumer thread 0..255
     uint32_t k = 0, sc = 0, cphase = 0;
     bool ok = true;
@@ -608,9 +716,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     bool pending = false;
     int pend_old = 0;     // thread 0: the unit counter before pd's partial was counted
     // The CTA that completes a unit merges its partials in slice order.
-    auto merge_unit = [&](const SegDesc &u) {
+    auto merge_unit = [&](const SegDesc &u, int first, int stride) {
         const int slot0 = u.unit + u.first;
-        for (int it = ct; it < G * (D / 8); it += kNumConsumerWarps * 32) {
+        for (int it = first; it < G * (D / 8); it += stride) {
             const int h = it / (D / 8), d0 = (it % (D / 8)) * 8;
             // One pass in slice order, rescaling the running sum as the max grows.
             float M = -INFINITY, L = 0.f;
@@ -652,7 +760,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         if (!consumer_sync(cons_bar, cphase, abort_flag))
             return false;
         if (*is_last_flag) {
-            merge_unit(pd);
+            merge_unit(pd, ct, kNumConsumerWarps * 32);
             // every partial of the unit has been counted: clear its counter for
             // the next attention launch over the same plan
             if (ct == 0)
@@ -684,6 +792,255 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                         p.lse[(size_t)b * p.num_q_heads + h] = -INFINITY;
             }
         }
+    }
+
+    if (warp_mode) {
+        // ======================== per-warp mode (short units) ========================
+        // Warp w of CTA c streams slice c * 8 + w alone, with its own stages
+        // (w + 8 m, m < S / 8), its own two query slots (w and w + 8) and its own
+        // merge tile, and ends each segment alone: no CTA barrier.  Lane 0 issues
+        // the copies, at most S / 8 pages and one segment ahead of the warp's
+        // consumption; each stage is used by this warp only, in order.
+        constexpr int R = S / kNumConsumerWarps;
+        static_assert(kSegRing >= 2 * kNumConsumerWarps, "two query slots per warp");
+        const long long slice = (long long)blockIdx.x * kNumConsumerWarps + warp;
+        if (slice >= T)
+            return;
+        const long long s0 = slice_begin(slice, W, T), s1 = slice_begin(slice + 1, W, T);
+        if (s0 >= s1)
+            return;
+        if (lane == 0) {
+            prefetch_tensor_map(&kmap);
+            prefetch_tensor_map(&vmap);
+        }
+        const uint64_t policy = l2_evict_first_policy();
+        const uint32_t q_bytes = (uint32_t)(G * D * 2);
+        float *tile = merge_o + (size_t)warp * kMaxGroup * C::kMergeStride;
+        float *tile_lse = merge_m + warp * kMaxGroup;
+
+        int bcur = warp_find_trajectory(p.page_prefix, p.batch, s0 / Hkv, lane);
+        // The segment that starts at flattened position x (trajectories without
+        // pages are skipped); se receives where it ends.
+        auto describe_at = [&](long long x, long long &se) -> SegDesc {
+            for (;;) {
+                const long long pb0 = p.page_prefix[bcur], pb1 = p.page_prefix[bcur + 1];
+                if (x >= pb1 * Hkv) {
+                    ++bcur;
+                    continue;
+                }
+                SegDesc d = describe_segment(x, bcur, pb0, pb1, s1, (int)slice, W, T, Hkv, se);
+                const int n = p.context_lens[bcur];
+                const int max_n = (int)((pb1 - pb0) * kPageSize);
+                d.n = n < max_n ? n : max_n;
+                return d;
+            }
+        };
+        uint32_t jw = 0, jc = 0;  // pages issued / consumed by this warp
+        uint32_t ki = 0, kc = 0;  // ordinals of the segments being issued / consumed
+        long long di_se, dc_se;
+        SegDesc di = describe_at(s0, di_se);
+        SegDesc dc = di;
+        dc_se = di_se;
+        int ii = 0;     // next page of di to issue
+        int cb = 0;     // first page of di whose table entry `chunk` holds
+        int chunk = 0;  // lane l: physical page of di's page cb + l
+        auto load_chunk = [&]() {
+            chunk = 0;
+            if (cb + lane < di.num_pages) {
+                chunk = __ldg(p.block_table + (size_t)di.b * p.max_pages + di.page_begin + cb + lane);
+                if (chunk < 0 || chunk >= p.num_pages) {
+                    record_status(&p.hdr->status, CADKV_ERR_OOB);
+                    chunk = 0;
+                }
+            }
+        };
+        auto load_q = [&](const SegDesc &d, uint32_t ord) {
+            if (lane == 0) {
+                const int slot = warp + kNumConsumerWarps * (int)(ord & 1u);
+                // the slot's previous query rows were read (generic proxy) before
+                // this copy (async proxy) overwrites them
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                mbar_arrive_expect_tx(&seg_full[slot], q_bytes);
+                bulk_load(qbuf + (size_t)slot * kMaxGroup * D,
+                          p.q + ((size_t)d.b * p.num_q_heads + (size_t)d.kvh * G) * D, q_bytes,
+                          &seg_full[slot]);
+            }
+        };
+        auto issue_more = [&]() {
+            while (jw - jc < (uint32_t)R) {
+                if (ii == di.num_pages) {
+                    if (ki != kc || di_se >= s1)
+                        break;  // already one segment ahead, or the slice ends here
+                    di = describe_at(di_se, di_se);
+                    ++ki;
+                    ii = 0;
+                    cb = 0;
+                    load_chunk();
+                    load_q(di, ki);
+                }
+                if (ii - cb == 32) {
+                    cb += 32;
+                    load_chunk();
+                }
+                const int phys = __shfl_sync(kFull, chunk, ii - cb);
+                // stage of page jw: its previous use (page jw - R) is consumed
+                const uint32_t st = warp + kNumConsumerWarps * (jw % R);
+                if (lane == 0) {
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    uint8_t *kdst = stages + (size_t)st * C::kStageBytes;
+                    uint8_t *vdst = kdst + C::kKBytes;
+                    const int ph_head = phys * Hkv + di.kvh;
+                    mbar_arrive_expect_tx(&full_bar[st], C::kStageBytes);
+                    if (C::kBoxes > 1 && p.whole_page_box) {
+                        tma_load_4d(kdst, &kmap, 0, 0, 0, ph_head, &full_bar[st], policy);
+                        tma_load_4d(vdst, &vmap, 0, 0, 0, ph_head, &full_bar[st], policy);
+                    } else {
+#pragma unroll
+                        for (int bx = 0; bx < C::kBoxes; ++bx) {
+                            tma_load_2d(kdst + bx * C::kBoxBytes, &kmap, bx * 64,
+                                        ph_head * kPageSize, &full_bar[st], policy);
+                            tma_load_2d(vdst + bx * C::kBoxBytes, &vmap, bx * 64,
+                                        ph_head * kPageSize, &full_bar[st], policy);
+                        }
+                    }
+                }
+                ++jw;
+                ++ii;
+            }
+        };
+
+        load_chunk();
+        load_q(di, 0);
+        issue_more();
+        bool wok = true;
+        for (;;) {
+            const int qslot = warp + kNumConsumerWarps * (int)(kc & 1u);
+            wok = __all_sync(kFull, mbar_wait(&seg_full[qslot], (kc >> 1) & 1u, abort_flag));
+            if (!wok)
+                break;
+            uint32_t qf[D / 16][2];
+            {
+                const __nv_bfloat16 *qs = qbuf + (size_t)qslot * kMaxGroup * D + g * D + 2 * t;
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    qf[kk][0] = *reinterpret_cast<const uint32_t *>(qs + 16 * kk);
+                    qf[kk][1] = *reinterpret_cast<const uint32_t *>(qs + 16 * kk + 8);
+                }
+            }
+            float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+            float o[D / 16][4];
+#pragma unroll
+            for (int mt = 0; mt < D / 16; ++mt)
+                o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+            for (int i = 0; i < dc.num_pages; ++i) {
+                const uint32_t st = warp + kNumConsumerWarps * (jc % R);
+                wok = __all_sync(kFull, mbar_wait(&full_bar[st], (jc / R) & 1u, abort_flag));
+                if (!wok)
+                    break;
+                const int valid = min(kPageSize, dc.n - (dc.page_begin + i) * kPageSize);
+                attend_page<D>(smem_addr(stages + (size_t)st * C::kStageBytes), valid, qf,
+                               p.scale_log2, m0, m1, l0, l1, o, lane);
+                __syncwarp();
+                ++jc;
+                issue_more();
+            }
+            if (!wok)
+                break;
+
+            // ---- the segment's result, from this warp alone
+#pragma unroll
+            for (int off = 4; off < 32; off <<= 1) {
+                l0 += __shfl_xor_sync(kFull, l0, off);
+                l1 += __shfl_xor_sync(kFull, l1, off);
+            }
+            {
+                const float inv0 = 1.f / l0, inv1 = 1.f / l1;
+#pragma unroll
+                for (int mt = 0; mt < D / 16; ++mt) {
+                    tile[(2 * t) * C::kMergeStride + 16 * mt + g] = o[mt][0] * inv0;
+                    tile[(2 * t + 1) * C::kMergeStride + 16 * mt + g] = o[mt][1] * inv1;
+                    tile[(2 * t) * C::kMergeStride + 16 * mt + g + 8] = o[mt][2] * inv0;
+                    tile[(2 * t + 1) * C::kMergeStride + 16 * mt + g + 8] = o[mt][3] * inv1;
+                }
+                if (g == 0) {
+                    tile_lse[2 * t] = m0 + __log2f(l0);
+                    tile_lse[2 * t + 1] = m1 + __log2f(l1);
+                }
+            }
+            __syncwarp();
+            const bool partial = dc.slot >= 0;
+            for (int it = lane; it < G * (D / 8); it += 32) {
+                const int h = it / (D / 8), d0 = (it % (D / 8)) * 8;
+                const float *src = tile + h * C::kMergeStride + d0;
+                const float lse2 = tile_lse[h];
+                if (!partial) {
+                    uint4 packed;
+                    packed.x = pack_bf16x2(src[0], src[1]);
+                    packed.y = pack_bf16x2(src[2], src[3]);
+                    packed.z = pack_bf16x2(src[4], src[5]);
+                    packed.w = pack_bf16x2(src[6], src[7]);
+                    const size_t row = (size_t)dc.b * p.num_q_heads + dc.kvh * G + h;
+                    *reinterpret_cast<uint4 *>(p.out + row * D + d0) = packed;
+                    if (d0 == 0 && p.lse)
+                        p.lse[row] = lse2 * kLn2;
+                } else {
+                    float4 *dst = reinterpret_cast<float4 *>(p.part_o + ((size_t)dc.slot * G + h) * D + d0);
+                    dst[0] = make_float4(src[0], src[1], src[2], src[3]);
+                    dst[1] = make_float4(src[4], src[5], src[6], src[7]);
+                    if (d0 == 0)
+                        p.part_lse[(size_t)dc.slot * G + h] = lse2;
+                }
+            }
+            __syncwarp();  // the tile is rewritten by the next segment; the partial is complete
+            if (partial) {
+                // count this partial (release: the warp's stores above, ordered by
+                // the warp barrier); the warp that completes the unit merges it
+                int old = 0;
+                if (lane == 0)
+                    asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], 1;"
+                                 : "=r"(old) : "l"(&p.unit_counter[dc.unit]) : "memory");
+                old = __shfl_sync(kFull, old, 0);
+                if (old == dc.count - 1) {
+                    __syncwarp();
+                    merge_unit(dc, lane, 32);
+                    if (lane == 0)
+                        p.unit_counter[dc.unit] = 0;
+                }
+            }
+
+            // ---- on to the next segment (the issuing side may have described it)
+            if (ki == kc) {
+                if (dc_se >= s1)
+                    break;
+                di = describe_at(dc_se, di_se);
+                ++ki;
+                ii = 0;
+                cb = 0;
+                load_chunk();
+                load_q(di, ki);
+            }
+            dc = di;
+            dc_se = di_se;
+            ++kc;
+            issue_more();
+        }
+        if (!wok) {
+            if (lane == 0) {
+                *abort_flag = 1;
+                record_status(&p.hdr->status, CADKV_ERR_TIMEOUT);
+                // every copy this warp started must land before it leaves
+                for (uint32_t j = jc; j < jw; ++j) {
+                    volatile int never = 0;
+                    mbar_wait(&full_bar[warp + kNumConsumerWarps * (j % R)], (j / R) & 1u, &never);
+                }
+                for (uint32_t o2 = kc; o2 <= ki; ++o2) {
+                    volatile int never = 0;
+                    mbar_wait(&seg_full[warp + kNumConsumerWarps * (int)(o2 & 1u)], (o2 >> 1) & 1u,
+                              &never);
+                }
+            }
+        }
+        return;
     }
 
     for (;;) {
@@ -726,88 +1083,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             ok = __all_sync(kFull, mbar_wait(&full_bar[st], (kk_idx / S) & 1, abort_flag));
             if (!ok)
                 break;
-            const uint32_t kbase = smem_addr(stages + (size_t)st * C::kStageBytes);
-            const uint32_t vbase = kbase + C::kKBytes;
             const int valid = min(kPageSize, d.n - (d.page_begin + i) * kPageSize);
-
-            // ---- S^T (16 tokens x 8 heads) = K (16 x D) . Q^T (D x 8)
-            float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
-            {
-                const int row = (mi & 1) * 8 + rr;
-#pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk) {
-                    const int chunk = 2 * kk + (mi >> 1);
-                    const uint32_t addr = kbase + (chunk >> 3) * C::kBoxBytes + row * 128 +
-                                          (((chunk & 7) ^ rr) << 4);
-                    uint32_t a0, a1, a2, a3;
-                    ldmatrix_x4(addr, a0, a1, a2, a3);
-                    if (kk & 1)
-                        mma_bf16_m16n8k16(sb, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
-                    else
-                        mma_bf16_m16n8k16(sa, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
-                }
-            }
-            // s[0]: (token g, head 2t)  s[1]: (g, 2t+1)  s[2]: (g+8, 2t)  s[3]: (g+8, 2t+1)
-            float s[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e)
-                s[e] = (sa[e] + sb[e]) * p.scale_log2;
-            if (valid < kPageSize) {
-                if (g >= valid) {
-                    s[0] = -INFINITY;
-                    s[1] = -INFINITY;
-                }
-                if (g + 8 >= valid) {
-                    s[2] = -INFINITY;
-                    s[3] = -INFINITY;
-                }
-            }
-            float mx0 = fmaxf(s[0], s[2]), mx1 = fmaxf(s[1], s[3]);
-#pragma unroll
-            for (int off = 4; off < 32; off <<= 1) {
-                mx0 = fmaxf(mx0, __shfl_xor_sync(kFull, mx0, off));
-                mx1 = fmaxf(mx1, __shfl_xor_sync(kFull, mx1, off));
-            }
-            const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-            const float alpha0 = exp2_approx(m0 - mn0), alpha1 = exp2_approx(m1 - mn1);
-            m0 = mn0;
-            m1 = mn1;
-            const float p0 = exp2_approx(s[0] - mn0), p1 = exp2_approx(s[1] - mn1);
-            const float p2 = exp2_approx(s[2] - mn0), p3 = exp2_approx(s[3] - mn1);
-            l0 = l0 * alpha0 + (p0 + p2);
-            l1 = l1 * alpha1 + (p1 + p3);
-#pragma unroll
-            for (int mt = 0; mt < D / 16; ++mt) {
-                o[mt][0] *= alpha0;
-                o[mt][1] *= alpha1;
-                o[mt][2] *= alpha0;
-                o[mt][3] *= alpha1;
-            }
-            // P^T as the B operand: transpose the two 8x8 (token x head) blocks.
-            const uint32_t pb0 = movmatrix_trans(pack_bf16x2(p0, p1));
-            const uint32_t pb1 = movmatrix_trans(pack_bf16x2(p2, p3));
-            uint32_t mask_lo = 0xffffffffu, mask_hi = 0xffffffffu;
-            if (valid < kPageSize) {  // zero value rows past n (they may hold NaN)
-                mask_lo = (2 * t < valid ? 0x0000ffffu : 0u) | (2 * t + 1 < valid ? 0xffff0000u : 0u);
-                mask_hi = (2 * t + 8 < valid ? 0x0000ffffu : 0u) | (2 * t + 9 < valid ? 0xffff0000u : 0u);
-            }
-            // ---- O^T (D x 8) += V^T (D x 16 tokens) . P^T (16 x 8)
-            {
-                const int row = (mi >> 1) * 8 + rr;
-#pragma unroll
-                for (int mt = 0; mt < D / 16; ++mt) {
-                    const int chunk = 2 * mt + (mi & 1);
-                    const uint32_t addr = vbase + (chunk >> 3) * C::kBoxBytes + row * 128 +
-                                          (((chunk & 7) ^ rr) << 4);
-                    uint32_t a0, a1, a2, a3;
-                    ldmatrix_x4_trans(addr, a0, a1, a2, a3);
-                    a0 &= mask_lo;
-                    a1 &= mask_lo;
-                    a2 &= mask_hi;
-                    a3 &= mask_hi;
-                    mma_bf16_m16n8k16(o[mt], a0, a1, a2, a3, pb0, pb1);
-                }
-            }
+            attend_page<D>(smem_addr(stages + (size_t)st * C::kStageBytes), valid, qf,
+                           p.scale_log2, m0, m1, l0, l1, o, lane);
             __syncwarp();
             if (lane == 0)
                 mbar_arrive(&empty_bar[st]);
@@ -943,7 +1221,8 @@ DecodeWorkspaceLayout decode_workspace_layout(int batch, int num_kv_heads, int g
 {
     DecodeWorkspaceLayout L{};
     L.slice_cap = num_sms * kSlicesPerCta;
-    L.capacity = batch * num_kv_heads + L.slice_cap;
+    L.capacity = batch * num_kv_heads +
+                 num_sms * (kSlicesPerCta > kNumConsumerWarps ? kSlicesPerCta : kNumConsumerWarps);
     size_t off = align_up(sizeof(WorkspaceHeader), kWorkspaceAlign);
     L.page_prefix = off;
     off = align_up(off + (size_t)(batch + 1) * sizeof(long long), kWorkspaceAlign);

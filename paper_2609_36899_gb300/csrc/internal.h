@@ -37,7 +37,8 @@ constexpr int kPageSize = 16;      // tokens per KV page
 constexpr int kMaxGroup = 8;       // query heads per KV head handled by one tile
 constexpr int kNumConsumerWarps = 8;
 constexpr int kAttnThreads = (kNumConsumerWarps + 1) * 32;
-constexpr int kSegRing = 8;        // segment descriptors in flight per CTA
+constexpr int kSegRing = 16;       // segment descriptors in flight per CTA (two per consumer
+                                   // warp in the per-warp mode)
 constexpr int kSlicesPerCta = 4;   // dynamic work slices per persistent CTA
 constexpr int kMinSlicePages = 16; // auto slicing never cuts finer than this
 constexpr long long kOneSliceMaxPerCta = 4096;  // page-heads per CTA up to which auto
@@ -48,6 +49,14 @@ constexpr size_t kWorkspaceAlign = 256;
 // the next decode step can launch while this step's attention kernel still
 // runs and wait there, and no attention CTA waits for an SM behind it.
 constexpr int kSmallPlanMaxBatch = 2048;
+// Per-warp mode: when the (trajectory, KV head) units are short, every consumer
+// warp streams a slice of its own (kNumConsumerWarps slices per CTA) and ends
+// its segments alone, instead of eight warps sharing each segment and merging
+// at its end.  Taken automatically when units average at most
+// kWarpModeMaxAvgPages pages and every warp slice gets at least
+// kWarpModeMinSlicePages page-heads.
+constexpr long long kWarpModeMaxAvgPages = 48;
+constexpr long long kWarpModeMinSlicePages = 4;
 
 // Work slices T of W flattened page-heads: one equal slice per CTA while a CTA
 // would hold at most kOneSliceMaxPerCta page-heads, up to kSlicesPerCta per CTA
@@ -77,7 +86,8 @@ struct alignas(64) WorkspaceHeader {
     long long dp_items;    // prefill: items run whole (the rest are split)
     long long pieces;      // prefill: pieces per split item
     long long first_segs;  // decode: CTAs whose first segment the planner described (0: none)
-    long long pad1;
+    int warp_mode;         // decode: 1 = per-warp slices (kNumConsumerWarps per CTA)
+    int pad1;
 };
 
 // Byte offsets of the decode-attention workspace regions.
@@ -91,7 +101,7 @@ struct DecodeWorkspaceLayout {
     size_t part_lse;      // fp32  [capacity][G]
     size_t part_o;        // fp32  [capacity][G][D]
     size_t total;
-    int capacity;         // partial slots = batch * Hkv + slice cap
+    int capacity;         // partial slots = batch * Hkv + the most slices of either mode
     int slice_cap;
 };
 

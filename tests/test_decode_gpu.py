@@ -382,10 +382,11 @@ def test_workspace_too_small_is_rejected():
     assert e.value.status == STATUS["CADKV_ERR_WORKSPACE"]
 
 
-@pytest.mark.parametrize("b,c", [(32, 16384), (8, 65536), (512, 1024)])
+@pytest.mark.parametrize("b,c", [(32, 16384), (8, 65536), (512, 1024), (512, 256),
+                                 (2048, 256)])
 def test_landscape_cells_every_row(b, c):
     """Cells of the (B, mean context) landscape sweep at full size, every row
-    against the oracle."""
+    against the oracle (the two cells of mean 256 take the per-warp mode)."""
     from paper_2609_36899_gb300.workloads import landscape_workload
     w = landscape_workload(b, c)
     batch = make_decode_batch(w, device="cuda")
