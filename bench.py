@@ -858,6 +858,11 @@ def main():
                     help="layers per chunk of the 48-layer staging job (default: the "
                          "largest that fits in device memory)")
     ap.add_argument("--staging-batch", type=int, default=None)
+    ap.add_argument("--landscape-batches", type=str, default=None,
+                    help="landscape: comma-separated batch sizes (default: the whole grid, "
+                         "with the composition cells)")
+    ap.add_argument("--landscape-means", type=str, default=None,
+                    help="landscape: comma-separated mean context lengths")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target oracle time of the cpu_baseline sample")
     ap.add_argument("--reference-seconds", type=float, default=90.0,
@@ -892,8 +897,13 @@ def main():
         # Composition cells (0.5-2 GB each) first, then the grid, whose cells grow
         # in size: no cell is allocated right after a much larger one was freed,
         # which left the next allocation's reads up to 30 % slower on this GPU.
-        comp = bench_composition(device, args.steps, args.warmup)
-        cells = bench_landscape(device, args.steps, args.warmup)
+        grid = {}
+        if args.landscape_batches:
+            grid["batches"] = tuple(int(x) for x in args.landscape_batches.split(","))
+        if args.landscape_means:
+            grid["means"] = tuple(int(x) for x in args.landscape_means.split(","))
+        comp = [] if grid else bench_composition(device, args.steps, args.warmup)
+        cells = bench_landscape(device, args.steps, args.warmup, **grid)
         if rank == 0:
             print(json.dumps({"workload": "decode-throughput landscape over (B, mean context), "
                                           "32/8 heads, D=128, lengths U[C/2, 3C/2]; and over the "
