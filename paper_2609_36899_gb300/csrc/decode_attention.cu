@@ -316,6 +316,17 @@ struct AttnConfig {
     static constexpr size_t kBytes = kFlagOff + 16 + 1024;  // + slack for 1024-B alignment
 };
 
+// A small-batch planner CTA (kPlanThreadsSmall threads) must fit on an SM beside an
+// attention CTA, so that the next step's planner can launch while this step's
+// attention kernel runs (see plan_kernel): shared memory of both, plus the 1 KB the
+// hardware reserves per CTA, within the SM's 228 KB.
+constexpr size_t kPlanSmemBytes = (size_t)(kSmallPlanMaxBatch + 1) * sizeof(long long) +
+                                  (size_t)kSmallPlanMaxBatch * sizeof(int) +
+                                  32 * sizeof(long long) + sizeof(long long);
+static_assert(AttnConfig<128>::kBytes + kPlanSmemBytes + 2 * 1024 <= 228 * 1024,
+              "the planner no longer fits beside an attention CTA");
+static_assert(AttnConfig<64>::kBytes <= AttnConfig<128>::kBytes, "D = 128 is the larger");
+
 // One page-head of a segment for one warp: S^T = K Q^T (16 tokens x 8 query
 // heads, mma.sync m16n8k16), online softmax over the page's valid tokens, and
 // O^T += V^T P^T.  kbase: the stage's K block (V follows it); tokens at or past
