@@ -188,14 +188,6 @@ __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::
                  "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])             \
                  : "memory")
 
-#define CADKV_TMEM_ST16(taddr, r)                                                                   \
-    asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,"    \
-                 "%11,%12,%13,%14,%15,%16};" ::"r"(taddr),                                        \
-                 "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]),       \
-                 "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]),   \
-                 "r"(r[14]), "r"(r[15])                                                           \
-                 : "memory")
-
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
@@ -803,11 +795,11 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                     const uint64_t nm2 = ((uint64_t)__float_as_uint(-m_use) << 32) | __float_as_uint(-m_use);
                     uint64_t l2 = 0;
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) {
-                        uint32_t packed[16];
+                    for (int c2 = 0; c2 < 2; ++c2) {
+                        uint32_t packed[32];
 #pragma unroll
-                        for (int e = 0; e < 32; e += 2) {
-                            const uint64_t x = ((uint64_t)r[32 * c + e + 1] << 32) | r[32 * c + e];
+                        for (int e = 0; e < 64; e += 2) {
+                            const uint64_t x = ((uint64_t)r[64 * c2 + e + 1] << 32) | r[64 * c2 + e];
                             uint64_t y;
                             asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(y) : "l"(x), "l"(sc2), "l"(nm2));
                             const float p0 = exp2_approx(__uint_as_float((uint32_t)y));
@@ -816,7 +808,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                             asm("add.f32x2 %0, %1, %2;" : "=l"(l2) : "l"(l2), "l"(pp));
                             packed[e >> 1] = pack_bf16x2(p0, p1);
                         }
-                        CADKV_TMEM_ST16(s_col + c * 16, packed);
+                        CADKV_TMEM_ST32(s_col + c2 * 32, packed);
                     }
                     lt = __uint_as_float((uint32_t)l2) + __uint_as_float((uint32_t)(l2 >> 32));
                     fresh = __any_sync(kFull, !(lt <= kMaxP));
@@ -837,11 +829,11 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                     const uint64_t nm2 = ((uint64_t)__float_as_uint(-m_use) << 32) | __float_as_uint(-m_use);
                     uint64_t l2 = 0;
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) {
-                        uint32_t packed[16];
+                    for (int c2 = 0; c2 < 2; ++c2) {
+                        uint32_t packed[32];
 #pragma unroll
-                        for (int e = 0; e < 32; e += 2) {
-                            const uint64_t x = ((uint64_t)r[32 * c + e + 1] << 32) | r[32 * c + e];
+                        for (int e = 0; e < 64; e += 2) {
+                            const uint64_t x = ((uint64_t)r[64 * c2 + e + 1] << 32) | r[64 * c2 + e];
                             uint64_t y;
                             asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(y) : "l"(x), "l"(sc2), "l"(nm2));
                             const float p0 = exp2_approx(__uint_as_float((uint32_t)y));
@@ -850,7 +842,7 @@ __global__ void __launch_bounds__(kPrefillThreads, 1)
                             asm("add.f32x2 %0, %1, %2;" : "=l"(l2) : "l"(l2), "l"(pp));
                             packed[e >> 1] = pack_bf16x2(p0, p1);
                         }
-                        CADKV_TMEM_ST16(s_col + c * 16, packed);
+                        CADKV_TMEM_ST32(s_col + c2 * 32, packed);
                     }
                     lt = __uint_as_float((uint32_t)l2) + __uint_as_float((uint32_t)(l2 >> 32));
                 }
