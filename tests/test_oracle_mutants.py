@@ -74,6 +74,18 @@ MUTANTS = [
      "const int64_t pos = row - q_offsets[b];", 1),
     ("prefill_gqa_interleaved", PREFILL, "const int64_t g = h / group;",
      "const int64_t g = h % num_kv_heads;", 1),
+    ("prefill_drop_softmax_scale", PREFILL,
+     "const double scale = 1.0 / sqrt((double)head_dim);", "const double scale = 1.0;", 1),
+    ("prefill_exponent_sign_flipped", PREFILL, "exp(s[t] - m)", "exp(m - s[t])", 1),
+    ("prefill_values_read_from_keys", PREFILL, "v_pages + ((phys", "k_pages + ((phys", 1),
+    ("prefill_normalised_by_length", PREFILL, "o[d] /= l;", "o[d] /= (double)n;", 1),
+    ("prefill_lse_without_max", PREFILL, "lse[i] = m + log(l);", "lse[i] = log(l);", 1),
+    ("prefill_key_slot_reversed", PREFILL,
+     "k_pages + ((phys * num_kv_heads + g) * page_size + t % page_size)",
+     "k_pages + ((phys * num_kv_heads + g) * page_size + (page_size - 1 - t % page_size))", 1),
+    ("prefill_query_of_next_head", PREFILL,
+     "q + (row * num_q_heads + h) * head_dim",
+     "q + (row * num_q_heads + (h + 1) % num_q_heads) * head_dim", 1),
 ]
 
 
