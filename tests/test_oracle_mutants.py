@@ -57,14 +57,26 @@ MUTANTS = [
     ("stage_wrong_layer", STAGE, "+ l * layer_stride", "+ (l - layer_begin) * layer_stride", 1),
     ("stage_packed_offset_one_layer", STAGE,
      "layers * 2 * num_kv_heads * head_dim", "2 * num_kv_heads * head_dim", 1),
+    ("stage_pool_head_reversed", STAGE,
+     "pool + ((phys * num_kv_heads + h) * page_size + slot)",
+     "pool + ((phys * num_kv_heads + (num_kv_heads - 1 - h)) * page_size + slot)", 1),
+    ("stage_dims_reversed", STAGE, "row[t * head_dim + d] = src[d];",
+     "row[t * head_dim + d] = src[head_dim - 1 - d];", 1),
     ("load_tokens_reversed", LOAD,
      "memcpy(d, row + t * head_dim", "memcpy(d, row + (n - 1 - t) * head_dim", 1),
     ("load_k_v_swapped", LOAD, "(kv == 0 ? k_pool : v_pool)", "(kv == 1 ? k_pool : v_pool)", 1),
+    ("load_pool_head_reversed", LOAD,
+     "pool + ((phys * num_kv_heads + h) * page_size + slot)",
+     "pool + ((phys * num_kv_heads + (num_kv_heads - 1 - h)) * page_size + slot)", 1),
     ("append_to_first_token", APPEND, "const int64_t t = n - 1;", "const int64_t t = 0;", 1),
     ("append_head_reversed", APPEND,
      "const int64_t src = (b * num_kv_heads + h) * head_dim;",
      "const int64_t src = (b * num_kv_heads + (num_kv_heads - 1 - h)) * head_dim;", 1),
     ("append_k_only", APPEND, "v_pages[dst + d] = v_new[src + d];", "", 1),
+    ("append_next_slot", APPEND, "const int64_t slot = t % page_size;",
+     "const int64_t slot = (t + 1) % page_size;", 1),
+    ("append_v_from_k", APPEND, "v_pages[dst + d] = v_new[src + d];",
+     "v_pages[dst + d] = k_new[src + d];", 1),
     ("prefill_excludes_own_token", PREFILL, "const int64_t n = pos + 1;",
      "const int64_t n = pos > 0 ? pos : 1;", 1),
     ("prefill_attends_whole_context", PREFILL, "const int64_t n = pos + 1;",
