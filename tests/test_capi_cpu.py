@@ -59,6 +59,8 @@ def _decode(lib, **over):
     (dict(batch=-1), "CADKV_ERR_SHAPE"),
     (dict(num_pages=0), "CADKV_ERR_SHAPE"),
     (dict(max_pages=-3), "CADKV_ERR_SHAPE"),
+    (dict(max_pages=1 << 27), "CADKV_ERR_SHAPE"),            # 16 * max_pages tokens overflow int32
+    (dict(num_pages=1 << 30), "CADKV_ERR_UNSUPPORTED"),      # page-head rows overflow int32
 ])
 def test_decode_attention_rejects_on_host(lib, over, code):
     assert _decode(lib, **over) == STATUS[code]
@@ -124,3 +126,5 @@ def test_prefill_rejects_on_host(lib):
     assert call(q=None) == STATUS["CADKV_ERR_INVALID"]
     assert call(offs=P((1 << 12) + 4)) == STATUS["CADKV_ERR_INVALID"]
     assert call(total=0) == 0
+    assert call(num_pages=1 << 30) == STATUS["CADKV_ERR_UNSUPPORTED"]
+    assert call(max_pages=1 << 27) == STATUS["CADKV_ERR_UNSUPPORTED"]
