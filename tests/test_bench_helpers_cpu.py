@@ -58,3 +58,30 @@ def test_profiled_traffic_follows_the_kernel_source(tmp_path):
     src.write_text("__global__ void k() { /* changed */ }\n")
     assert bench.profiled_traffic(str(summary), str(src)) is None
     assert bench.profiled_traffic(str(tmp_path / "missing.md"), str(src)) is None
+
+
+def test_reference_arm_prints_the_contract_line():
+    """``bench.py --impl reference`` (the fp64 oracle on the host cores) prints one
+    JSON line carrying the keys the benchmark contract asks of that arm."""
+    import json
+    import os
+    import subprocess
+    import sys
+    from pathlib import Path
+    root = Path(__file__).resolve().parents[1]
+    r = subprocess.run([sys.executable, str(root / "bench.py"), "--impl", "reference",
+                        "--workload", "tiny", "--steps", "3", "--warmup", "3",
+                        "--reference-seconds", "1"],
+                       capture_output=True, text=True, timeout=300, cwd=root,
+                       env={**os.environ, "CUDA_VISIBLE_DEVICES": ""})
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    line = json.loads(lines[0])
+    assert line["impl"] == "reference" and line["unit"] == "GB/s" and line["value"] > 0
+    assert line["higher_is_better"] is True and line["steps"] == 3 and line["warmup"] == 3
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+    assert line["cpu_baseline"]["value"] == line["value"]
+    assert line["e2e"] == {"value": line["value"], "unit": "GB/s", "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
+    assert line["config"]["workload"] == "tiny decode attention"
